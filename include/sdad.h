@@ -285,6 +285,18 @@ sdad_status sdad_workspace_init(void* ws, void* stream);
  * (outputs of that call are then unspecified), or SDAD_ERR_CUDA. */
 sdad_status sdad_check(void* ws, void* stream);
 
+/* Sets how many times each bounded device wait of the calls that use `ws`
+ * polls before it gives up (Sec. 5 of the paper has no counterpart: this is
+ * failure detection of the GPU path).  polls < 0 restores the default
+ * (2^22 polls); 0 <= polls < 2^32 - 1 sets that limit, 0 meaning that every
+ * wait gives up at once.  A wait that gives up records SDAD_ERR_TIMEOUT
+ * (read by sdad_check); the kernel still waits, with the default limit, for
+ * the copies and tensor-core work it issued itself before it returns.
+ * Enqueued on `stream` (a one-thread kernel writes the header field);
+ * sdad_workspace_init restores the default.
+ * Errors: SDAD_ERR_NULL, SDAD_ERR_ALIGN, SDAD_ERR_SHAPE, SDAD_ERR_CUDA. */
+sdad_status sdad_workspace_set_wait_limit(void* ws, int64_t polls, void* stream);
+
 /* ========================================================================
  * Loss + gradient entry points.  All pointers are device pointers.
  * ======================================================================== */
@@ -438,15 +450,23 @@ sdad_status sdad_batax_grad(const sdad_csr* A, const float* X, float beta, float
                             const int32_t* jrowptr, const int32_t* jcolidx, int64_t jnnz,
                             float* J_val, void* ws, size_t ws_bytes, void* stream);
 
-/* Least squares exactly as sdad_lsq_grad, for callers that cannot allocate
- * device memory or pass a workspace (for example code running under a memory
+/* Least squares as sdad_lsq_grad, for callers that cannot allocate device
+ * memory or pass a workspace (for example code running under a memory
  * allocator it does not own, such as a framework's caching pool or a host
  * that reserves all device memory at start-up).  The paper has no
  * counterpart; this is a deployment convenience.
+ *   Layouts: the plain CSR, and in SDAD_T_CSC / AUTO mode with dx the plain
+ *   CSC twin (colptr, rowidx, val_csc).  The ranked column numbering and a
+ *   row-blocked twin are ignored; a matrix that carries a row-blocked twin
+ *   but no plain CSC twin for every column (a split twin, or a blocked twin
+ *   alone) is refused in CSC mode with SDAD_ERR_UNSUPPORTED, although
+ *   sdad_lsq_grad accepts it.
  *   Scratch: a fixed 8 MiB array compiled into the library, present on every
- *   device that loads it until the process exits.  A problem whose scratch
- *   (sdad_workspace_bytes for SDAD_EXPR_LSQ) exceeds 8 MiB is rejected with
- *   SDAD_ERR_WORKSPACE before any device work.
+ *   device that loads it until the process exits.  A problem needs about
+ *   66 KiB + 4 m + 12 nnz / 256 bytes of it (each region rounded up to 256
+ *   bytes); one that needs more than 8 MiB is rejected with
+ *   SDAD_ERR_WORKSPACE before any device work (at 50M keys that leaves room
+ *   for about 1.49M rows).
  *   The call allocates nothing (no cudaMalloc/cudaFree).  Its first call on a
  *   device looks up the array's device address (cudaGetSymbolAddress); make
  *   that first call before any stream capture.  Each call clears the part of

@@ -60,6 +60,8 @@ sdad_status check_device() {
   return ok_cache[dev] == 1 ? SDAD_OK : SDAD_ERR_UNSUPPORTED;
 }
 
+__global__ void set_wait_kernel(WsHeader* h, uint32_t v) { h->wait_polls = v; }
+
 __global__ void zero_kernel(float* __restrict__ p, size_t n) {
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n;
        i += (size_t)gridDim.x * blockDim.x)
@@ -238,6 +240,15 @@ sdad_status sdad_workspace_init(void* ws, void* stream) {
   if (!ws) return SDAD_ERR_NULL;
   if ((reinterpret_cast<uintptr_t>(ws) & 255) != 0) return SDAD_ERR_ALIGN;
   return map_cuda(cudaMemsetAsync(ws, 0, sizeof(WsHeader), (cudaStream_t)stream));
+}
+
+sdad_status sdad_workspace_set_wait_limit(void* ws, int64_t polls, void* stream) {
+  if (!ws) return SDAD_ERR_NULL;
+  if ((reinterpret_cast<uintptr_t>(ws) & 255) != 0) return SDAD_ERR_ALIGN;
+  if (polls >= (int64_t)0xFFFFFFFFll) return SDAD_ERR_SHAPE;
+  const uint32_t v = polls < 0 ? 0u : (uint32_t)polls + 1u;
+  set_wait_kernel<<<1, 1, 0, (cudaStream_t)stream>>>(static_cast<WsHeader*>(ws), v);
+  return map_cuda(cudaGetLastError());
 }
 
 sdad_status sdad_check(void* ws, void* stream) {

@@ -22,7 +22,8 @@ constexpr unsigned FULL_MASK = 0xffffffffu;
 struct WsHeader {
   int32_t status;       // sticky error code (0 = ok), cleared by sdad_check
   uint32_t ticket;      // last-CTA ticket of the loss reduction, back to 0 after use
-  uint32_t pad[62];
+  uint32_t wait_polls;  // 0: bounded waits poll kWaitPolls times; v > 0: v - 1 times
+  uint32_t pad[61];
 };
 static_assert(sizeof(WsHeader) == 256, "header is 256 bytes");
 
@@ -93,9 +94,29 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 
 // Polls at most kWaitPolls times (each poll may suspend the thread for a
 // short, hardware-chosen time), then records a timeout and returns false.
+// The workspace header can lower the limit (sdad_workspace_set_wait_limit),
+// down to no poll at all, so that the timeout path can be exercised.
 constexpr uint32_t kWaitPolls = 1u << 22;
 
+__device__ __forceinline__ uint32_t wait_limit(const WsHeader* h) {
+  const uint32_t v = *reinterpret_cast<const volatile uint32_t*>(&h->wait_polls);
+  return v ? v - 1 : kWaitPolls;
+}
+
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, WsHeader* h) {
+  const uint32_t lim = wait_limit(h);
+  for (uint32_t it = 0; it < lim; ++it)
+    if (mbar_try_wait(bar, parity)) return true;
+  set_status(h, SDAD_ERR_TIMEOUT);
+  return false;
+}
+
+// The wait a kernel makes before it returns, for asynchronous work it issued
+// itself (bulk copies into its shared memory, MMAs into its tensor memory):
+// always the full kWaitPolls limit, whatever the header asks, so that a
+// kernel that gave up on an earlier wait does not leave while its own copies
+// are still landing.  Records a timeout if even that runs out.
+__device__ __forceinline__ bool mbar_drain(uint64_t* bar, uint32_t parity, WsHeader* h) {
   for (uint32_t it = 0; it < kWaitPolls; ++it)
     if (mbar_try_wait(bar, parity)) return true;
   set_status(h, SDAD_ERR_TIMEOUT);

@@ -205,6 +205,7 @@ __device__ __forceinline__ double run_pipeline(const StreamSrc<NARR>& src, Body&
     // ---------------- producer ----------------
     PtrWindow pw{src.ptr, src.nseg + 1, sm.pwin, -1, src.side, sm.swin};
     int lb_cs = 0;   // lower_bound(ptr, cs), carried from the previous chunk
+    int issued = 0;  // chunks whose stage this warp has filled (copies issued, arrival made)
     for (int c = c0; c < c1; ++c) {
       const int k = c - c0;
       const int s = k % NS;
@@ -278,7 +279,12 @@ __device__ __forceinline__ double run_pipeline(const StreamSrc<NARR>& src, Body&
       }
       __syncwarp();
       lb_cs = lb_ce;
+      issued = k + 1;
     }
+    // the copies of the last NS stages may still be landing (consumers that
+    // gave up on a wait do not consume them): wait for each before leaving
+    for (int k = max(0, issued - NS); k < issued; ++k)
+      if (!mbar_drain(&sm.full[k % NS], (k / NS) & 1, hdr)) break;
   } else {
     // ---------------- consumers ----------------
     for (int c = c0; c < c1; ++c) {

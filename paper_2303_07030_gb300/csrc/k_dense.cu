@@ -144,8 +144,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     }
     // all threads take the same decision (a wait that gave up ends the kernel)
     const bool got = __syncthreads_and(mbar_wait(&S.bar_load, ph_load, hdr));
+    if (!got) {   // the tile's copy may still be landing: let it, then leave
+      mbar_drain(&S.bar_load, ph_load, hdr);
+      break;
+    }
     ph_load ^= 1;
-    if (!got) break;
     // split the tile in place: hi stays, lo goes to the twin buffer
     {
       float4* hi4 = reinterpret_cast<float4*>(&S.a_hi[0][0]);
@@ -178,8 +181,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
       tc::mma_commit(&S.bar_mma);
     }
     const bool done = __syncthreads_and(mbar_wait(&S.bar_mma, ph_mma, hdr));
+    if (!done) {   // the MMAs still write tensor memory: let them end before it is freed
+      mbar_drain(&S.bar_mma, ph_mma, hdr);
+      break;
+    }
     ph_mma ^= 1;
-    if (!done) break;
     tc::fence_after_sync();
     // epilogue: warp w owns tile rows 32w .. 32w+31 (its TMEM lane quadrant)
     {

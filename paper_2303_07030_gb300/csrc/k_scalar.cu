@@ -829,13 +829,10 @@ cudaError_t bcol_pass(const sdad_csr* A, const float* rvec, float* out, const Ws
   const size_t smem = sizeof(float) << lg;
   cudaError_t e;
   if (split && (e = col_pass(A, A->bcsc_rest_nnz, rvec, out, L, st)) != cudaSuccess) return e;
-  static bool attr = false;
-  if (!attr) {
-    e = cudaFuncSetAttribute(scalar_bcol_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)(sizeof(float) << SDAD_BCSC_MAX_LOG2));
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
+  // the limit belongs to the device: raised once per (kernel, device)
+  e = ensure_dynamic_smem(reinterpret_cast<const void*>(scalar_bcol_kernel),
+                          (int)(sizeof(float) << SDAD_BCSC_MAX_LOG2));
+  if (e != cudaSuccess) return e;
   const int sms = device_sm_count();
   if (nchunks > 0) {
     int per_sm = 1;

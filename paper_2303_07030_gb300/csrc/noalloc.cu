@@ -68,6 +68,9 @@ extern "C" sdad_status sdad_lsq_grad_noalloc(const sdad_csr* A, const float* x, 
   // nor the row-blocked twin; a CSC twin that holds only some columns (the
   // rest of a split twin) cannot serve the column pass alone
   if (csc && csr_split(A)) return SDAD_ERR_UNSUPPORTED;
+  // a matrix that carries only a row-blocked twin (no plain CSC twin) has no
+  // column structure this entry point can read
+  if (csc && csr_blocked(A) && !A->colptr) return SDAD_ERR_UNSUPPORTED;
   plain.bcsc_log2 = 0;
   plain.bcsc_cols = nullptr;
   sdad_status s = check_csr(A, csc);

@@ -32,6 +32,7 @@ EXPORTS = [
     "sdad_status_string", "sdad_version", "sdad_csr_from_coo", "sdad_csr_transpose",
     "sdad_csr_rank_columns", "sdad_csr_block_transpose", "sdad_csr_transpose_rest",
     "sdad_coo3_mode_index", "sdad_workspace_bytes", "sdad_workspace_init", "sdad_check",
+    "sdad_workspace_set_wait_limit",
     "sdad_lsq_grad", "sdad_logreg_grad", "sdad_mf_grad", "sdad_cp3_grad", "sdad_gnn_grad",
     "sdad_lsq_grad_noalloc", "sdad_lsq_jvp", "sdad_logreg_jvp", "sdad_mf_jvp", "sdad_cp3_jvp",
     "sdad_smvm_grad", "sdad_smmm_grad", "sdad_csr_gram_pattern",
@@ -95,6 +96,7 @@ def lib():
             "sdad_workspace_bytes": ([i32, i32, i32, i64, i32, P(sz)], i32),
             "sdad_workspace_init": ([vp, vp], i32),
             "sdad_check": ([vp, vp], i32),
+            "sdad_workspace_set_wait_limit": ([vp, i64, vp], i32),
             "sdad_lsq_grad": ([P(sdad_csr), vp, vp, vp, vp, vp, i32, vp, sz, vp], i32),
             "sdad_logreg_grad": ([P(sdad_csr), vp, vp, vp, vp, vp, i32, vp, sz, vp], i32),
             "sdad_mf_grad": ([P(sdad_csr), vp, vp, i32, f32, vp, vp, vp, vp, i32, vp, sz, vp],
@@ -267,6 +269,12 @@ def sdad_workspace_init(ws, stream=None):
 
 def sdad_check(ws, stream=None):
     return lib().sdad_check(_ptr(ws), _stream(stream))
+
+
+def sdad_workspace_set_wait_limit(ws, polls, stream=None):
+    """polls < 0: the default limit; otherwise every bounded wait polls that often."""
+    _check(lib().sdad_workspace_set_wait_limit(_ptr(ws), int(polls), _stream(stream)),
+           "sdad_workspace_set_wait_limit")
 
 
 class Workspace:

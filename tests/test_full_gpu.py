@@ -31,15 +31,21 @@ def _problem_and_oracle(name):
     return _cache[name]
 
 
-# the logistic cases: the benchmark's default (ranked columns), the split
-# column pass (blocked columns with >= 32 keys per 2^15-row block), the atomic
-# transposed product, and the columns as generated
+# the logistic cases: the layout the benchmark times (ranked columns and a
+# row-blocked CSC twin of every column with 2^15-row blocks: 31 blocks), the
+# ranked columns with the plain CSC twin, the split column pass (blocked
+# columns with >= 32 keys per 2^15-row block), the atomic transposed product,
+# and the columns as generated; CP with its one-pass atomic scatter (AUTO) and
+# with the sorted per-mode passes (SDAD_T_CSC)
 @pytest.mark.parametrize("name,kw", [
+    ("logreg", {"ranked": True, "blocked": 15}),
     ("logreg", {"ranked": True}),
     ("logreg", {"ranked": True, "split": (15, 32.0)}),
     ("logreg", {"ranked": True, "tmode": 2}),
     ("logreg", {}),
-    ("mf", {}), ("cp3", {}), ("gnn", {}),
+    ("mf", {}),
+    ("cp3", {}), ("cp3", {"tmode": 1}),
+    ("gnn", {}),
 ])
 def test_full_size_parity(name, kw):
     p, ref = _problem_and_oracle(name)
