@@ -1,18 +1,22 @@
 #!/usr/bin/env python3
-"""Benchmark: loss + full gradient of a sparse loss on one GB300 per rank.
+"""Benchmark: loss + full gradient of sparse losses on one GB300 per rank.
 
-Default workload: sparse logistic regression, X 1,000,000 x 100,000 CSR with
-~50 keys per row (Poisson row lengths, Zipf(1.1) column ids, lognormal
-values), labels Bernoulli(0.5), w ~ N(0, 0.01); one step = one call of
-sdad_logreg_grad (loss and dL/dw) with every input resident in HBM.
-``--config`` selects another of the five workloads (lsq, logreg, mf, cp3,
-gnn) at full size.
+Headline workload (the largest): graph propagation Y = A (H W), L = 1/2
+|Y - Z|^2 on an R-MAT graph of 2^22 vertices and 2^26 edges (a, b, c = .57,
+.19, .19), H 2^22 x 128, W 128 x 64; one step = one call of sdad_gnn_grad
+(loss, dA on A's keys, dH, dW) with every input resident in HBM.  The line
+also carries, under "configs", the same measurement of every other workload
+(least squares, logistic regression, matrix factorisation, CP, and the
+paper's SMVM, SMMM and BATAX kernels), each at full size, and the FP32 FMA
+rate measured in the same run ("fp32_fma_peak"), against which the
+arithmetic-bound kernels are reported.  ``--config`` picks another headline;
+``--others none`` measures the headline alone.
 
 Prints one JSON line (rank 0).  Timing: W warm-up steps, then K steps, each
 bracketed by CUDA events on the launching stream; the inputs of the large
-workloads exceed the 129 MB L2, the small least-squares workload flushes L2
-(writes 256 MB) between timed steps.  Per-kernel times come from the
-library's event records of the same timed steps.
+workloads exceed the 129 MB L2, the small workloads flush L2 (a 256 MB write)
+between timed steps.  Per-kernel times come from a second pass of the same
+K steps with every library kernel bracketed by events on its stream.
 
 ``--impl reference`` times the fp64 CPU oracle instead (host cores, bounded
 sample of the same workload); under torchrun only rank 0 runs it.
@@ -52,13 +56,20 @@ WORKLOAD_NAMES = {
 }
 
 
+ALL_CONFIGS = ["gnn", "logreg", "mf", "cp3", "lsq", "smvm", "smmm", "batax"]
+SMALL_CONFIGS = ("lsq", "smvm", "smmm", "batax")   # inputs below L2: flushed between steps
+
+
 def parse():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--config", default="logreg", choices=list(WORKLOAD_NAMES))
+    ap.add_argument("--config", default="gnn", choices=list(WORKLOAD_NAMES),
+                    help="the headline workload (default: the largest, graph propagation)")
+    ap.add_argument("--others", default="all", choices=["all", "none"],
+                    help="all: also measure every other workload under the line's 'configs'")
     ap.add_argument("--tmode", default="auto", choices=["auto", "csc", "atomic"])
     ap.add_argument("--transpose", default="auto", choices=["auto", "csc", "blocked", "split"],
                     help="lsq/logreg: column pass over the plain CSC twin; over a row-blocked "
@@ -77,8 +88,8 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--override", action="append", default=[], metavar="KEY=VALUE",
-                    help="change a generator parameter of the workload (profiling of a "
-                         "smaller instance, e.g. m=400000); the line then says so")
+                    help="change a generator parameter of the headline workload (profiling of "
+                         "a smaller instance, e.g. m=400000); the line then says so")
     return ap.parse_args()
 
 
@@ -165,33 +176,54 @@ def kernel_bytes(cfg, p, nnz, tmode_csc, want_extra, ranked=False, blocked=0, sp
     return b
 
 
+def kernel_flops(cfg, p, nnz):
+    """FP32 arithmetic per launch of the kernels bound by it rather than by HBM."""
+    f = {}
+    if cfg == "mf":
+        f["mf_row"] = 256 * nnz       # per key: 64-wide dot (128) + 64-wide axpy (128)
+        f["mf_col"] = 256 * nnz
+        f["mf_atomic"] = 384 * nnz    # dot + two axpys (dU in registers, dV scattered)
+    elif cfg == "cp3":
+        f["cp_atomic"] = 384 * nnz    # e: 32 x 3; three 32-wide gradient terms: 3 x 32 x 3
+        f["cp_mode"] = 192 * nnz      # e and one mode's gradient term
+    elif cfg == "gnn":
+        f["proj_dw"] = 2 * p.n * 128 * 64
+    return f
+
+
 # ----------------------------------------------------------------------------
 # measured DRAM traffic (ncu dram__bytes_read.sum + dram__bytes_write.sum) of
-# the logistic passes, per key, from one capture of the 400,000-row instance
-# (20,000,407 keys; see profiles/logreg_passes.md) in the bench's default
-# layout (ranked columns, row-blocked CSC twin of 2^15-row blocks), scaled to
-# a launch by its keys.  The figure belongs to the kernel source it was taken
-# on: when that file changes, or the layout differs, the traffic is reported
-# as null until it is captured again.
+# some kernels, per key, each from one capture of a reduced instance of its
+# workload in the benchmark's layout, scaled to a launch by its keys (traffic
+# grows with the keys at fixed density).  A figure belongs to the kernel
+# source it was taken on: when that file changes, or the layout differs, the
+# traffic is reported as null until it is captured again.
 # ----------------------------------------------------------------------------
 NCU_TRAFFIC = {
-    "source": "paper_2303_07030_gb300/csrc/k_scalar.cu",
-    "sha1": "0dbc677f8113ea28c84b7c761a8184b5ebfb8195",
-    "layout": {"ranked": True, "blocked": 15, "split": False},
-    "bytes_per_key": {"logreg_row": 8.5676, "scalar_bcol": 8.4912},
+    "logreg": {
+        # 400,000-row instance, 20,000,407 keys; ranked columns, 2^15-row blocked twin
+        "source": "paper_2303_07030_gb300/csrc/k_scalar.cu",
+        "sha1": "0dbc677f8113ea28c84b7c761a8184b5ebfb8195",
+        "layout": {"ranked": True, "blocked": 15, "split": False},
+        "bytes_per_key": {"logreg_row": 8.5676, "scalar_bcol": 8.4912},
+        "capture": "ncu capture of the 400k-row instance, scaled by keys",
+    },
 }
 
 
-def measured_traffic(kernel, nnz):
+def measured_traffic(cfg, kernel, nnz, layout=None):
     import hashlib
+    ent = NCU_TRAFFIC.get(cfg)
+    if ent is None or (ent.get("layout") is not None and layout != ent["layout"]):
+        return None, None
     try:
-        with open(os.path.join(ROOT, NCU_TRAFFIC["source"]), "rb") as f:
-            if hashlib.sha1(f.read()).hexdigest() != NCU_TRAFFIC["sha1"]:
-                return None
+        with open(os.path.join(ROOT, ent["source"]), "rb") as f:
+            if hashlib.sha1(f.read()).hexdigest() != ent["sha1"]:
+                return None, None
     except OSError:
-        return None
-    b = NCU_TRAFFIC["bytes_per_key"].get(kernel)
-    return None if b is None else int(round(b * nnz))
+        return None, None
+    b = ent["bytes_per_key"].get(kernel)
+    return (None, None) if b is None else (int(round(b * nnz)), ent["capture"])
 
 
 # ----------------------------------------------------------------------------
@@ -383,32 +415,28 @@ def torch_empty_pinned_like(t):
     return torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
 
 
-def main():
-    args = parse()
-    rank = int(os.environ.get("RANK", "0"))
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
+def fp32_fma_peak(S, torch, stream):
+    """FP32 FMA rate of this GPU (TFLOP/s): best of five probe launches."""
+    sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+    blocks, iters = sms * 8, 8192
+    out = torch.empty(blocks * 256, dtype=torch.float32, device="cuda")
+    S.sdad_probe_fma(out, blocks, iters, stream)   # warm-up
+    best = None
+    for _ in range(5):
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        fl = S.sdad_probe_fma(out, blocks, iters, stream)
+        b.record(stream)
+        torch.cuda.synchronize()
+        t = a.elapsed_time(b) * 1e-3
+        best = t if best is None else min(best, t)
+    return {"tflops": round(fl / best / 1e12, 2), "how": "%d CTAs x 256 threads, 16 independent "
+            "FMA chains of %d steps per thread, best of 5 (CUDA events)" % (blocks, iters)}
 
-    if args.impl == "reference":
-        if rank != 0:
-            return 0
-        return run_reference(args)
 
-    import torch
-    torch.cuda.set_device(local)
-    dist = None
-    if world > 1:
-        import torch.distributed as dist
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-
-    from paper_2303_07030_gb300 import build as B
-    from paper_2303_07030_gb300 import sdad as S
-    from paper_2303_07030_gb300 import workloads as W
-    B.build()
-
-    cfg = args.config
-    ov = overrides(args)
-    p = W.make(cfg, "full", **ov)
+def layout_for(cfg, p, args, S):
+    """(ranked, blocked, block_cols, split, transpose) of a workload's matrix."""
     ranked = cfg in ("lsq", "logreg") and (
         args.columns == "ranked" or (args.columns == "auto" and cfg == "logreg"))
     blocked, block_cols, split = 0, None, None
@@ -421,13 +449,25 @@ def main():
         if transpose == "split":
             block_cols = S.split_columns(p.col, p.n, p.m, blocked, args.block_min)
             split = (int(block_cols.size), int(np.isin(p.col, block_cols).sum()))
-    run = make_run(cfg, p, args.tmode, ranked, blocked, block_cols)
+    return ranked, blocked, block_cols, split, transpose
+
+
+def measure(cfg, args, ov, dist, world, local, headline, fma):
+    """One workload: timed steps, per-kernel times, rooflines; e2e for the headline."""
+    import torch
+    from paper_2303_07030_gb300 import sdad as S
+    from paper_2303_07030_gb300 import workloads as W
+
+    p = W.make(cfg, "full", **ov)
+    ranked, blocked, block_cols, split, transpose = layout_for(cfg, p, args, S)
+    tmode = args.tmode if headline else "auto"
+    run = make_run(cfg, p, tmode, ranked, blocked, block_cols)
     if cfg == "batax":
         p.params["jnnz"] = run.jnnz
     nnz = step_keys(cfg, p)
     stream = torch.cuda.current_stream()
     flush = None
-    if cfg == "lsq":
+    if cfg in SMALL_CONFIGS:
         flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
 
     def barrier():
@@ -491,31 +531,38 @@ def main():
         a = per.setdefault(name, [0, 0.0])
         a[0] += 1
         a[1] += kms
-    csc = getattr(run, "csc", args.tmode != "atomic")
+    csc = getattr(run, "csc", tmode != "atomic")
     kb = kernel_bytes(cfg, p, nnz, csc, False, ranked, blocked, split)
+    kf = kernel_flops(cfg, p, nnz)
     dom = max((k for k in per if k in kb), key=lambda k: per[k][1], default=None)
     hbm, src = peaks()
     roofline = None
     if dom is not None:
         avg_ms = per[dom][1] / per[dom][0]
         ach = kb[dom] / (avg_ms * 1e-3) / 1e9
+        layout = {"ranked": ranked, "blocked": blocked, "split": split is not None}
+        traffic, tsrc = measured_traffic(cfg, dom, nnz, layout)
         roofline = {"bound": "hbm", "kernel": dom, "achieved": round(ach, 1), "peak": hbm,
                     "peak_source": src, "unit": "GB/s", "frac": round(ach / hbm, 4),
-                    "traffic": measured_traffic(dom, nnz)
-                    if cfg == "logreg" and NCU_TRAFFIC["layout"] == {
-                        "ranked": ranked, "blocked": blocked, "split": split is not None}
-                    else None,
-                    "traffic_source": "ncu capture of the 400k-row instance, scaled by keys"
-                    if cfg == "logreg" else None,
-                    "algorithmic_bytes": kb[dom],
-                    "avg_launch_ms": round(avg_ms, 5)}
-    kernels = {k: {"launches": v[0], "ms_per_launch": round(v[1] / v[0], 5),
-                   "share": round(v[1] / max(sum(x[1] for x in per.values()), 1e-12), 4)}
-               for k, v in per.items()}
+                    "traffic": traffic, "traffic_source": tsrc,
+                    "algorithmic_bytes": kb[dom], "avg_launch_ms": round(avg_ms, 5)}
+    tot_ms = max(sum(x[1] for x in per.values()), 1e-12)
+    kernels = {}
+    for k, v in per.items():
+        e = {"launches": v[0], "ms_per_launch": round(v[1] / v[0], 5),
+             "share": round(v[1] / tot_ms, 4)}
+        if k in kb:
+            gbs = kb[k] / (v[1] / v[0] * 1e-3) / 1e9
+            e["hbm_frac"] = round(gbs / hbm, 4)
+        if k in kf and fma:
+            tf = kf[k] / (v[1] / v[0] * 1e-3) / 1e12
+            e["fp32_tflops"] = round(tf, 2)
+            e["fp32_frac"] = round(tf / fma["tflops"], 4)
+        kernels[k] = e
 
     # ---------------- end to end: host buffers, copies inside the timing ----
     e2e = None
-    if not args.no_e2e:
+    if headline and not args.no_e2e:
         ins = host_inputs(run, cfg)
         outs = host_outputs(run, cfg)
         h2d = sum(h.numel() * h.element_size() for _, h in ins)
@@ -539,6 +586,7 @@ def main():
                 h.copy_(d, non_blocking=True)
         e1.record(stream)
         torch.cuda.synchronize()
+        run.check()
         ems = e0.elapsed_time(e1) / args.steps
         if dist is not None:
             t = torch.tensor([ems], device="cuda", dtype=torch.float64)
@@ -546,36 +594,91 @@ def main():
             ems = float(t.item())
         e2e = {"value": world * nnz / (ems * 1e-3), "unit": UNIT, "ms_per_step": round(ems, 4),
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+        del ins, outs
+    tot = sum(kb.get(k, 0) * v[0] for k, v in per.items()) / max(args.steps, 1)
+    res = {
+        "value": value, "ms_per_step": round(ms, 5),
+        "config": {"workload": WORKLOAD_NAMES[cfg] + (" (overridden: %s)" % ov if ov else ""),
+                   "name": cfg, "nnz": nnz, "tmode": tmode,
+                   "columns": ("ranked by key count" if ranked else "as generated")
+                   if cfg in ("lsq", "logreg") else None,
+                   "transpose": transpose_name(blocked, split)
+                   if cfg in ("lsq", "logreg") else None,
+                   "l2": ("L2 flushed (256 MB write) between timed steps" if flush is not None
+                          else "inputs larger than L2 (no flush)"),
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "roofline": roofline, "kernels": kernels,
+        "ms_per_step_kernels_bracketed": round(bracketed_ms, 5),
+        "gpu_launches": int(len(recs)), "launches_per_step": len(recs) / max(args.steps, 1),
+        "hbm_gbs_step": round(tot / (ms * 1e-3) / 1e9, 1), "clocks": clocks, "e2e": e2e,
+    }
+    del run, flush
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    return p, res
 
+
+def main():
+    args = parse()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        if rank != 0:
+            return 0
+        return run_reference(args)
+
+    import torch
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    from paper_2303_07030_gb300 import build as B
+    from paper_2303_07030_gb300 import sdad as S
+    B.build()
+
+    stream = torch.cuda.current_stream()
+    fma = fp32_fma_peak(S, torch, stream)
+    cfg = args.config
+    ov = overrides(args)
+    p, head = measure(cfg, args, ov, dist, world, local, True, fma)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(cfg, p)
+    del p
+    others = {}
+    if args.others == "all":
+        for c in ALL_CONFIGS:
+            if c == cfg:
+                continue
+            q, r = measure(c, args, {}, dist, world, local, False, fma)
+            del q
+            others[c] = {k: r[k] for k in ("value", "ms_per_step", "roofline", "kernels",
+                                           "gpu_launches", "hbm_gbs_step", "clocks")}
+            others[c]["workload"] = r["config"]["workload"]
+            others[c]["nnz"] = r["config"]["nnz"]
+            if r["config"]["transpose"]:
+                others[c]["transpose"] = r["config"]["transpose"]
+                others[c]["columns"] = r["config"]["columns"]
 
     if rank == 0:
-        launches_per_step = len(recs) / max(args.steps, 1)
         line = {
-            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 5),
+            "metric": METRIC, "value": head["value"], "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": head["ms_per_step"],
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
             "data": "synthetic (seeded generators; no external dataset)",
-            "config": {"workload": WORKLOAD_NAMES[cfg] + (" (overridden: %s)" % ov if ov else ""),
-                       "name": cfg, "nnz": nnz,
-                       "tmode": args.tmode,
-                       "columns": ("ranked by key count" if ranked else "as generated")
-                       if cfg in ("lsq", "logreg") else None,
-                       "transpose": transpose_name(blocked, split)
-                       if cfg in ("lsq", "logreg") else None,
-                       "l2": ("L2 flushed (256 MB write) between timed steps" if flush is not None
-                              else "inputs larger than L2 (no flush)"),
-                       "parallelism": "replicas" if world > 1 else "single GPU"},
-            "roofline": roofline, "kernels": kernels,
-            "ms_per_step_kernels_bracketed": round(bracketed_ms, 5),
-            "gpu_launches": int(len(recs)), "launches_per_step": launches_per_step,
-            "hbm_gbs_step": None,
-            "clocks": clocks, "e2e": e2e, "cpu_baseline": cpu,
+            "config": head["config"], "roofline": head["roofline"], "kernels": head["kernels"],
+            "ms_per_step_kernels_bracketed": head["ms_per_step_kernels_bracketed"],
+            "gpu_launches": head["gpu_launches"],
+            "gpu_launches_all_configs": head["gpu_launches"] + sum(
+                o["gpu_launches"] for o in others.values()),
+            "launches_per_step": head["launches_per_step"],
+            "hbm_gbs_step": head["hbm_gbs_step"], "clocks": head["clocks"], "e2e": head["e2e"],
+            "cpu_baseline": cpu, "fp32_fma_peak": fma, "configs": others,
         }
-        tot = sum(kb.get(k, 0) * v[0] for k, v in per.items()) / max(args.steps, 1)
-        line["hbm_gbs_step"] = round(tot / (ms * 1e-3) / 1e9, 1)
         print(json.dumps(line), flush=True)
     if dist is not None:
         dist.barrier()

@@ -492,6 +492,17 @@ int32_t sdad_timing_count(void);
  * SDAD_ERR_NULL, SDAD_ERR_CUDA. */
 sdad_status sdad_timing_get(int32_t i, const char** name, float* ms);
 
+/* Measurement aid (the paper has no counterpart): enqueues a kernel of
+ * `blocks` CTAs x 256 threads, each thread running 16 independent FP32 FMA
+ * chains `iters` steps long, and stores the FLOPs it performs in *flops
+ * (host).  Timed by the caller with events on `stream`, it gives the FP32
+ * FMA rate against which the arithmetic-bound kernels are reported.
+ *   out[blocks*256]  device, overwritten (keeps the work observable)
+ * Errors: SDAD_ERR_NULL, SDAD_ERR_SHAPE (blocks or iters <= 0),
+ * SDAD_ERR_UNSUPPORTED (not sm_103), SDAD_ERR_CUDA. */
+sdad_status sdad_probe_fma(float* out, int32_t blocks, int32_t iters, double* flops,
+                           void* stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -38,6 +38,7 @@ EXPORTS = [
     "sdad_smvm_grad", "sdad_smmm_grad", "sdad_csr_gram_pattern",
     "sdad_batax_grad",
     "sdad_timing_enable", "sdad_timing_reset", "sdad_timing_count", "sdad_timing_get",
+    "sdad_probe_fma",
 ]
 
 
@@ -119,6 +120,7 @@ def lib():
             "sdad_timing_reset": ([], i32),
             "sdad_timing_count": ([], i32),
             "sdad_timing_get": ([i32, P(ctypes.c_char_p), P(ctypes.c_float)], i32),
+            "sdad_probe_fma": ([vp, i32, i32, P(ctypes.c_double), vp], i32),
         }
         for name, (args, res) in sigs.items():
             fn = getattr(L, name)
@@ -317,6 +319,14 @@ def sdad_timing_get(i):
 def sdad_timing_records():
     """All (kernel name, milliseconds) records since the last reset."""
     return [sdad_timing_get(i) for i in range(sdad_timing_count())]
+
+
+def sdad_probe_fma(out, blocks, iters, stream=None):
+    """Enqueues the FP32 FMA probe; returns the FLOPs it performs."""
+    fl = ctypes.c_double(0.0)
+    _check(lib().sdad_probe_fma(_ptr(out), int(blocks), int(iters), ctypes.byref(fl),
+                                _stream(stream)), "sdad_probe_fma")
+    return fl.value
 
 
 # ----------------------------------------------------------------------------

@@ -66,3 +66,31 @@ def test_reference_arm_prints_one_json_line():
     assert d["impl"] == "reference" and d["metric"] == bench.METRIC and d["value"] > 0
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["cpu_baseline"]["kind"] == "oracle"
     assert d["steps"] == 2 and d["warmup"] == 1
+
+
+def test_flops_and_traffic_tables():
+    p = W.make("mf", "small")
+    f = bench.kernel_flops("mf", p, p.nnz)
+    assert f["mf_row"] == 256 * p.nnz and f["mf_atomic"] == 384 * p.nnz
+    g = W.make("gnn", "small")
+    assert bench.kernel_flops("gnn", g, g.nnz)["proj_dw"] == 2 * g.n * 128 * 64
+    # a figure is given only for the layout it was captured on
+    lay = dict(bench.NCU_TRAFFIC["logreg"]["layout"])
+    t, src = bench.measured_traffic("logreg", "logreg_row", 1000, lay)
+    assert (t is None) == (src is None)
+    lay["blocked"] = 0
+    assert bench.measured_traffic("logreg", "logreg_row", 1000, lay) == (None, None)
+    assert bench.measured_traffic("lsq", "lsq_row", 1000, None) == (None, None)
+
+
+def test_default_headline_is_the_largest_workload():
+    sizes = {"gnn": 1 << 26, "logreg": 49_997_656, "mf": 50_000_000, "cp3": 10_000_000}
+    assert max(sizes, key=sizes.get) == "gnn"
+    sys_argv = sys.argv
+    try:
+        sys.argv = ["bench.py"]
+        a = bench.parse()
+    finally:
+        sys.argv = sys_argv
+    assert a.config == "gnn" and a.others == "all"
+    assert set(bench.ALL_CONFIGS) == set(bench.WORKLOAD_NAMES)
