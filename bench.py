@@ -149,6 +149,9 @@ def kernel_bytes(cfg, p, nnz, tmode_csc, want_extra, ranked=False, blocked=0, sp
         k = 64
         b["mf_row"] = 8 * nnz + 4 * (m + 1) + 4 * k * (m + n) + 4 * k * m
         b["mf_col"] = 8 * nnz + 4 * (n + 1) + 4 * k * (m + n) + 4 * k * n
+        # one pass: column ids, ranks and values of the keys; U, V read; dU, dV written
+        b["mf_atomic"] = 12 * nnz + 4 * (m + 1) + 2 * 4 * k * (m + n)
+        b["mf_init"] = 2 * 4 * k * (m + n)
     elif cfg == "cp3":
         d = sum(p.dims)
         b["cp_mode"] = 12 * nnz + 4 * (max(p.dims) + 1) + 4 * 32 * d + 4 * 32 * max(p.dims)
@@ -186,8 +189,6 @@ def kernel_flops(cfg, p, nnz):
     elif cfg == "cp3":
         f["cp_atomic"] = 384 * nnz    # e: 32 x 3; three 32-wide gradient terms: 3 x 32 x 3
         f["cp_mode"] = 192 * nnz      # e and one mode's gradient term
-    elif cfg == "gnn":
-        f["proj_dw"] = 2 * p.n * 128 * 64
     return f
 
 
@@ -382,8 +383,8 @@ def make_run(cfg, p, tmode, ranked, blocked=0, block_cols=None):
         return R.LsqRun(p, tmode=tm, ranked=ranked, blocked=blocked, block_cols=block_cols)
     if cfg == "logreg":
         return R.LogregRun(p, tmode=tm, ranked=ranked, blocked=blocked, block_cols=block_cols)
-    if cfg == "mf":
-        return R.MfRun(p)
+    if cfg == "mf":   # ranked columns: the atomic scatter sums the hot ones in shared memory
+        return R.MfRun(p, tmode=tm, ranked=True)
     if cfg == "cp3":
         return R.Cp3Run(p, tmode=tm)
     if cfg in ("smvm", "smmm", "batax"):

@@ -187,6 +187,24 @@ sdad_status sdad_coo3_mode_index(int64_t nnz, const int32_t* i, const int32_t* j
                                  const int32_t* k, const int32_t dims[3], int32_t mode,
                                  int32_t* perm, int32_t* segptr);
 
+/* Device gather of 32-bit words through a permutation: out[q] = src[perm[q]]
+ * for q < count, and 0 where perm[q] is outside [0, n_src) (the -1 that
+ * sdad_csr_block_transpose writes for padding keys).  It forms, on the
+ * device and on `stream`, the value copies that the physical formats hold
+ * beside the CSR values (Sec. 5.3: one dictionary, several storages):
+ *   val_csc  = gather(val, perm of sdad_csr_transpose / _transpose_rest)
+ *   bcsc_val = gather(val, bperm of sdad_csr_block_transpose)
+ *   sval[m], sidx[m][c] = gather(val, idx[c]; perm_m of sdad_coo3_mode_index)
+ * so a caller whose sparse values change between calls (a step that updates
+ * A itself) refreshes the twins without a host round trip.  The index arrays
+ * of the twins do not change with the values.
+ *   src[n_src], perm[count], out[count]: device, 16-byte aligned; out must not
+ *   overlap src or perm.
+ * Errors: SDAD_ERR_NULL, SDAD_ERR_SHAPE, SDAD_ERR_ALIGN, SDAD_ERR_UNSUPPORTED
+ * (not sm_103), SDAD_ERR_CUDA. */
+sdad_status sdad_gather_by_perm(const void* src, int64_t n_src, const int32_t* perm,
+                                int64_t count, void* out, void* stream);
+
 /* ========================================================================
  * Device operands (non-owning descriptors of device arrays)
  * ======================================================================== */
@@ -398,6 +416,20 @@ sdad_status sdad_mf_jvp(const sdad_csr* R, const float* U, const float* V, int32
 sdad_status sdad_cp3_jvp(const sdad_coo3* T, const float* A, const float* B, const float* C,
                          int32_t rank, const float* T_t_val, const float* A_t, const float* B_t,
                          const float* C_t, double* loss, double* loss_t, void* ws,
+                         size_t ws_bytes, void* stream);
+
+/* Forward mode of the graph propagation loss (f_in = 128, f_out = 64):
+ *   L = 1/2 |A (H W) - Z|^2 and its directional derivative L' along a tangent
+ *   of A's values (A_t_val on keys(A), CSR order), of H (H_t, n x 128) and of
+ *   W (W_t, 128 x 64), by the tensorized forward rules of Sec. 4.2 with a
+ *   real tangent: P' = H' W + H W' (tensor cores, as P), Y' = A' P + A P',
+ *   L' = sum_i (Y_i - Z_i) . Y'_i.  Every tangent is nullable (zero); dense
+ *   arrays 16-byte aligned.  One pass over the CSR (no CSC twin needed).
+ *   Workspace: as sdad_gnn_grad.  Reproducible bit for bit.
+ * Errors: NULL/SHAPE/ALIGN/OVERFLOW/WORKSPACE/CUDA/UNSUPPORTED (widths). */
+sdad_status sdad_gnn_jvp(const sdad_csr* A, const float* H, const float* W, const float* Z,
+                         int32_t f_in, int32_t f_out, const float* A_t_val, const float* H_t,
+                         const float* W_t, double* loss, double* loss_t, void* ws,
                          size_t ws_bytes, void* stream);
 
 /* ========================================================================

@@ -62,6 +62,18 @@ sdad_status check_device() {
 
 __global__ void set_wait_kernel(WsHeader* h, uint32_t v) { h->wait_polls = v; }
 
+// out[q] = src[perm[q]] for q < count (32-bit words); perm entries outside
+// [0, n_src) (the -1 of padding keys) give 0
+__global__ void gather32_kernel(const uint32_t* __restrict__ src, int64_t n_src,
+                                const int32_t* __restrict__ perm, int64_t count,
+                                uint32_t* __restrict__ out) {
+  for (int64_t q = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; q < count;
+       q += (int64_t)gridDim.x * blockDim.x) {
+    const int32_t p = __ldg(perm + q);
+    out[q] = (p >= 0 && p < n_src) ? __ldg(src + p) : 0u;
+  }
+}
+
 __global__ void zero_kernel(float* __restrict__ p, size_t n) {
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n;
        i += (size_t)gridDim.x * blockDim.x)
@@ -146,6 +158,9 @@ WsLayout ws_layout(int expr, int32_t rows, int32_t cols, int64_t nnz, int32_t wi
     L.D = reinterpret_cast<float*>(take(sizeof(float) * (size_t)std::max(rows, 1) * f));
     L.G = reinterpret_cast<float*>(take(sizeof(float) * (size_t)std::max(cols, 1) * f));
     L.dWpart = reinterpret_cast<float*>(take(sizeof(float) * (size_t)kDwParts * 128 * f));
+    const size_t nch = (size_t)(std::max<int64_t>(nnz, 0) / kMinCap + 2);
+    L.tfirst = reinterpret_cast<float*>(take(sizeof(float) * nch * f));
+    L.tlast = reinterpret_cast<float*>(take(sizeof(float) * nch * f));
   }
   const bool scalar = expr == SDAD_EXPR_LSQ || expr == SDAD_EXPR_LOGREG ||
                       expr == SDAD_EXPR_SMVM || expr == SDAD_EXPR_SMMM || expr == SDAD_EXPR_BATAX;
@@ -203,6 +218,74 @@ sdad_status check_ws(const WsLayout& need, void* ws, size_t ws_bytes) {
   return SDAD_OK;
 }
 
+// ---------------------------------------------------------------------------
+// SDAD_T_AUTO: the transposed product chosen by measured throughput
+// ---------------------------------------------------------------------------
+// An operand is identified by its device, expression, two of its device
+// pointers, its sizes and the outputs asked for.  The first AUTO call on it
+// runs the call in both modes, twice each, times the second run of each with
+// events on the call's stream (so it waits for the stream) and keeps the
+// faster; later AUTO calls on the same operand run the kept mode only.  A
+// call made while the stream is being captured into a graph does no timing:
+// it runs `fallback` (a choice made earlier is still used).
+struct AutoKey {
+  int dev, expr;
+  const void* a;
+  const void* b;
+  int64_t nnz;
+  int32_t m, n;
+  uint32_t flags;
+  bool operator==(const AutoKey& o) const {
+    return dev == o.dev && expr == o.expr && a == o.a && b == o.b && nnz == o.nnz && m == o.m &&
+           n == o.n && flags == o.flags;
+  }
+};
+
+namespace {
+std::mutex g_auto_mu;
+std::vector<std::pair<AutoKey, sdad_tmode>> g_auto;
+}  // namespace
+
+template <class Run>
+cudaError_t run_auto(AutoKey key, sdad_tmode fallback, cudaStream_t st, Run run) {
+  if (cudaGetDevice(&key.dev) != cudaSuccess) return cudaErrorInvalidDevice;
+  {
+    std::lock_guard<std::mutex> lock(g_auto_mu);
+    for (const auto& kv : g_auto)
+      if (kv.first == key) return run(kv.second);
+  }
+  cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+  cudaError_t e = cudaStreamIsCapturing(st, &cap);
+  if (e != cudaSuccess) return e;
+  if (cap != cudaStreamCaptureStatusNone) return run(fallback);
+  cudaEvent_t ev[2];
+  if ((e = cudaEventCreate(&ev[0])) != cudaSuccess) return e;
+  if ((e = cudaEventCreate(&ev[1])) != cudaSuccess) {
+    cudaEventDestroy(ev[0]);
+    return e;
+  }
+  const sdad_tmode modes[2] = {SDAD_T_CSC, SDAD_T_ATOMIC};
+  float ms[2] = {0.f, 0.f};
+  for (int trial = 0; trial < 2 && e == cudaSuccess; ++trial)
+    for (int k = 0; k < 2 && e == cudaSuccess; ++k) {
+      if ((e = cudaEventRecord(ev[0], st)) != cudaSuccess) break;
+      if ((e = run(modes[k])) != cudaSuccess) break;
+      if ((e = cudaEventRecord(ev[1], st)) != cudaSuccess) break;
+      if ((e = cudaEventSynchronize(ev[1])) != cudaSuccess) break;
+      if (trial == 1) e = cudaEventElapsedTime(&ms[k], ev[0], ev[1]);
+    }
+  cudaEventDestroy(ev[0]);
+  cudaEventDestroy(ev[1]);
+  if (e != cudaSuccess) return e;
+  // the outputs are those of the last run (ATOMIC), a complete evaluation
+  const sdad_tmode pick = ms[0] <= ms[1] ? SDAD_T_CSC : SDAD_T_ATOMIC;
+  std::lock_guard<std::mutex> lock(g_auto_mu);
+  bool found = false;
+  for (const auto& kv : g_auto) found = found || kv.first == key;
+  if (!found) g_auto.emplace_back(key, pick);
+  return cudaSuccess;
+}
+
 }  // namespace sdad
 
 using namespace sdad;
@@ -242,6 +325,23 @@ sdad_status sdad_workspace_init(void* ws, void* stream) {
   return map_cuda(cudaMemsetAsync(ws, 0, sizeof(WsHeader), (cudaStream_t)stream));
 }
 
+sdad_status sdad_gather_by_perm(const void* src, int64_t n_src, const int32_t* perm,
+                                int64_t count, void* out, void* stream) {
+  if (n_src < 0 || count < 0) return SDAD_ERR_SHAPE;
+  if (count == 0) return SDAD_OK;
+  if (!perm || !out || (n_src > 0 && !src)) return SDAD_ERR_NULL;
+  if (!a16(perm) || !a16(out) || (src && !a16(src))) return SDAD_ERR_ALIGN;
+  sdad_status s;
+  if ((s = check_device())) return s;
+  const int grid = (int)std::min<int64_t>((count + 255) / 256, (int64_t)device_sm_count() * 8);
+  {
+    KTimer t("gather_by_perm", (cudaStream_t)stream);
+    gather32_kernel<<<grid, 256, 0, (cudaStream_t)stream>>>(
+        static_cast<const uint32_t*>(src), n_src, perm, count, static_cast<uint32_t*>(out));
+  }
+  return map_cuda(cudaGetLastError());
+}
+
 sdad_status sdad_workspace_set_wait_limit(void* ws, int64_t polls, void* stream) {
   if (!ws) return SDAD_ERR_NULL;
   if ((reinterpret_cast<uintptr_t>(ws) & 255) != 0) return SDAD_ERR_ALIGN;
@@ -271,9 +371,12 @@ static sdad_status scalar_entry(int expr, const sdad_csr* A, const float* xin, c
                                 size_t ws_bytes, void* stream) {
   if (tmode < SDAD_T_AUTO || tmode > SDAD_T_ATOMIC) return SDAD_ERR_SHAPE;
   if (!A) return SDAD_ERR_NULL;
-  const bool csc = scalar_uses_csc(A, dvec != nullptr, tmode);
   const bool blocked = csr_blocked(A);
   const bool split = csr_split(A);
+  // AUTO without a column structure for every column: the atomic scatter
+  if (tmode == SDAD_T_AUTO && dvec && (blocked ? split && !A->colptr : !A->colptr))
+    tmode = SDAD_T_ATOMIC;
+  const bool csc = scalar_uses_csc(A, dvec != nullptr, tmode);
   sdad_status s = check_csr(A, csc && !blocked);
   if (s) return s;
   if (blocked) {
@@ -307,7 +410,15 @@ static sdad_status scalar_entry(int expr, const sdad_csr* A, const float* xin, c
   const WsLayout L = ws_layout(expr, A->m, A->n, A->nnz, blocked ? A->bcsc_log2 : 0, ws);
   if ((s = check_ws(L, ws, ws_bytes))) return s;
   if ((s = check_device())) return s;
-  return map_cuda(run_scalar(expr, A, xin, y, loss, dvec, dA, tmode, L, (cudaStream_t)stream));
+  const cudaStream_t st = (cudaStream_t)stream;
+  auto run = [&](sdad_tmode mode) { return run_scalar(expr, A, xin, y, loss, dvec, dA, mode, L, st); };
+  if (tmode == SDAD_T_AUTO && dvec) {
+    const uint32_t flags = 1u | (dA ? 2u : 0u) | (blocked ? 4u : 0u) | (split ? 8u : 0u) |
+                           (csr_ranked(A) ? 16u : 0u);
+    return map_cuda(run_auto(AutoKey{0, expr, A->rowptr, A->colidx, A->nnz, A->m, A->n, flags},
+                             SDAD_T_CSC, st, run));
+  }
+  return map_cuda(run(tmode));
 }
 
 sdad_status sdad_lsq_grad(const sdad_csr* A, const float* x, const float* y, double* loss,
@@ -326,17 +437,33 @@ sdad_status sdad_mf_grad(const sdad_csr* R, const float* U, const float* V, int3
                          float lambda, double* loss, float* dU, float* dV, float* dR_val,
                          sdad_tmode tmode, void* ws, size_t ws_bytes, void* stream) {
   if (tmode < SDAD_T_AUTO || tmode > SDAD_T_ATOMIC) return SDAD_ERR_SHAPE;
-  if (tmode == SDAD_T_ATOMIC) return SDAD_ERR_UNSUPPORTED;
   if (k != 64) return SDAD_ERR_UNSUPPORTED;
-  sdad_status s = check_csr(R, dV != nullptr);
+  if (!R) return SDAD_ERR_NULL;
+  // AUTO without the CSC twin: the one-pass atomic scatter
+  if (tmode == SDAD_T_AUTO && dV && !R->colptr) tmode = SDAD_T_ATOMIC;
+  sdad_status s = check_csr(R, dV != nullptr && tmode != SDAD_T_ATOMIC);
   if (s) return s;
+  if (csr_ranked(R)) {   // used by the atomic scatter (hot columns in shared memory)
+    if ((R->n > 0 && !R->rankcol) || (R->nnz > 0 && !R->rcolidx)) return SDAD_ERR_NULL;
+    if (R->nnz > 0 && !a16(R->rcolidx)) return SDAD_ERR_ALIGN;
+  }
   if (!U || !V || !loss) return SDAD_ERR_NULL;
   if (!a16(U) || !a16(V) || (dU && !a16(dU)) || (dV && !a16(dV)) || !a8(loss))
     return SDAD_ERR_ALIGN;
   const WsLayout L = ws_layout(SDAD_EXPR_MF, R->m, R->n, R->nnz, k, ws);
   if ((s = check_ws(L, ws, ws_bytes))) return s;
   if ((s = check_device())) return s;
-  return map_cuda(run_mf(R, U, V, lambda, loss, dU, dV, dR_val, tmode, L, (cudaStream_t)stream));
+  const cudaStream_t st = (cudaStream_t)stream;
+  auto run = [&](sdad_tmode mode) {
+    return run_mf(R, U, V, lambda, loss, dU, dV, dR_val, mode, L, st);
+  };
+  if (tmode == SDAD_T_AUTO && dV) {
+    const uint32_t flags = 1u | (dU ? 2u : 0u) | (dR_val ? 4u : 0u) | (csr_ranked(R) ? 8u : 0u);
+    return map_cuda(run_auto(AutoKey{0, SDAD_EXPR_MF, R->rowptr, R->colidx, R->nnz, R->m, R->n,
+                                     flags},
+                             SDAD_T_CSC, st, run));
+  }
+  return map_cuda(run(tmode == SDAD_T_ATOMIC ? SDAD_T_ATOMIC : SDAD_T_CSC));
 }
 
 sdad_status sdad_cp3_grad(const sdad_coo3* T, const float* A, const float* B, const float* C,
@@ -353,14 +480,13 @@ sdad_status sdad_cp3_grad(const sdad_coo3* T, const float* A, const float* B, co
   float* dfac[3] = {dA, dB, dC};
   for (int m = 0; m < 3; ++m)
     if (dfac[m] && !a16(dfac[m])) return SDAD_ERR_ALIGN;
-  // AUTO: the one-pass atomic scatter (measured faster on the CP workload)
-  // when the entry-order arrays are given, else the sorted per-mode passes
-  if (tmode == SDAD_T_AUTO)
-    tmode = (T->nnz == 0 || (T->idx[0] && T->idx[1] && T->idx[2] && T->val)) ? SDAD_T_ATOMIC
-                                                                            : SDAD_T_CSC;
-  if (tmode == SDAD_T_ATOMIC) {
+  // the entry-order arrays (one-pass atomic scatter) ...
+  auto check_entries = [&]() -> sdad_status {
     if (T->nnz > 0 && (!T->idx[0] || !T->idx[1] || !T->idx[2] || !T->val)) return SDAD_ERR_NULL;
-  } else {
+    return SDAD_OK;
+  };
+  // ... and the sorted copies of the modes asked for (per-mode passes)
+  auto check_sorted = [&]() -> sdad_status {
     int first = -1;
     for (int m = 0; m < 3; ++m) {
       const bool used = dfac[m] != nullptr || (first < 0 && m == 0 && !dA && !dB && !dC);
@@ -372,13 +498,32 @@ sdad_status sdad_cp3_grad(const sdad_coo3* T, const float* A, const float* B, co
       if (!a16(T->sidx[m][o1]) || !a16(T->sidx[m][o2]) || !a16(T->sval[m])) return SDAD_ERR_ALIGN;
     }
     if (dT_val && T->nnz > 0 && !T->sperm[first]) return SDAD_ERR_NULL;
+    return SDAD_OK;
+  };
+  sdad_status s;
+  bool measure = false;
+  if (tmode == SDAD_T_AUTO) {
+    // both layouts given: chosen by measured throughput; else the one given
+    const bool ent = check_entries() == SDAD_OK, srt = check_sorted() == SDAD_OK;
+    measure = ent && srt && T->nnz > 0;
+    tmode = ent ? SDAD_T_ATOMIC : SDAD_T_CSC;
   }
+  if ((s = tmode == SDAD_T_ATOMIC ? check_entries() : check_sorted())) return s;
   const int32_t dmax = std::max(T->dims[0], std::max(T->dims[1], T->dims[2]));
   const WsLayout L = ws_layout(SDAD_EXPR_CP3, dmax, dmax, T->nnz, rank, ws);
-  sdad_status s = check_ws(L, ws, ws_bytes);
-  if (s) return s;
+  if ((s = check_ws(L, ws, ws_bytes))) return s;
   if ((s = check_device())) return s;
-  return map_cuda(run_cp3(T, A, B, C, loss, dA, dB, dC, dT_val, tmode, L, (cudaStream_t)stream));
+  const cudaStream_t st = (cudaStream_t)stream;
+  auto run = [&](sdad_tmode mode) {
+    return run_cp3(T, A, B, C, loss, dA, dB, dC, dT_val, mode, L, st);
+  };
+  if (measure) {
+    const uint32_t flags = (dA ? 1u : 0u) | (dB ? 2u : 0u) | (dC ? 4u : 0u) | (dT_val ? 8u : 0u);
+    return map_cuda(run_auto(AutoKey{0, SDAD_EXPR_CP3, T->idx[0], T->segptr[0], T->nnz,
+                                     T->dims[0], T->dims[1], flags ^ ((uint32_t)T->dims[2] << 4)},
+                             SDAD_T_ATOMIC, st, run));
+  }
+  return map_cuda(run(tmode));
 }
 
 static sdad_status jvp_entry(int expr, const sdad_csr* A, const float* v, const float* y,
@@ -512,6 +657,24 @@ sdad_status sdad_gnn_grad(const sdad_csr* A, const float* H, const float* W, con
   if ((s = check_ws(L, ws, ws_bytes))) return s;
   if ((s = check_device())) return s;
   return map_cuda(run_gnn(A, H, W, Z, loss, dA_val, dH, dW, L, (cudaStream_t)stream));
+}
+
+sdad_status sdad_gnn_jvp(const sdad_csr* A, const float* H, const float* W, const float* Z,
+                         int32_t f_in, int32_t f_out, const float* A_t_val, const float* H_t,
+                         const float* W_t, double* loss, double* loss_t, void* ws,
+                         size_t ws_bytes, void* stream) {
+  if (f_in != 128 || f_out != 64) return SDAD_ERR_UNSUPPORTED;
+  sdad_status s = check_csr(A, false);
+  if (s) return s;
+  if (!H || !W || !Z || !loss || !loss_t) return SDAD_ERR_NULL;
+  for (const float* f : {H, W, Z, H_t, W_t})
+    if (f && !a16(f)) return SDAD_ERR_ALIGN;
+  if (!a8(loss) || !a8(loss_t)) return SDAD_ERR_ALIGN;
+  const WsLayout L = ws_layout(SDAD_EXPR_GNN, A->m, A->n, A->nnz, f_out, ws);
+  if ((s = check_ws(L, ws, ws_bytes))) return s;
+  if ((s = check_device())) return s;
+  return map_cuda(run_gnn_jvp(A, H, W, Z, A_t_val, H_t, W_t, loss, loss_t, L,
+                              (cudaStream_t)stream));
 }
 
 sdad_status sdad_timing_enable(int32_t on) {

@@ -135,6 +135,23 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       : "memory");
 }
 
+// Asynchronous 16-byte global->shared copy (cp.async, L2 only): `bytes` of
+// the 16 are read (0..16), the rest of the destination is zero-filled.  Both
+// addresses 16-byte aligned.  Completion: cp_async_commit / cp_async_wait.
+__device__ __forceinline__ void cp_async16_zfill(void* dst, const void* src, uint32_t bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)), "l"(src),
+               "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+// Waits until at most N of this thread's committed groups are pending.
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+
 // Hint to bring elements [b, e) of a 4-byte array into L2 (bulk prefetch by
 // the copy engine; no registers, no completion).  Only whole 16-byte units
 // inside the range are named, so nothing outside the array is touched.

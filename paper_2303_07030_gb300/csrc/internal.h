@@ -37,6 +37,8 @@ struct WsLayout {
   float* D;           // graph: A (H W) - Z                        [rows x f_out]
   float* G;           // graph: A^T D                              [cols x f_out]
   float* dWpart;      // graph: per-CTA partial H^T G              [kDwParts x f_in x f_out]
+  float* tfirst;      // graph, forward mode: pieces of Y' (as pfirst / plast below)
+  float* tlast;
   // pieces of segments cut by chunk boundaries (deterministic combination):
   float* pfirst;      // per chunk: the piece of the segment begun in an earlier chunk
   float* plast;       // per chunk: the piece of the segment that continues past it
@@ -109,6 +111,10 @@ cudaError_t run_mf(const sdad_csr* R, const float* U, const float* V, float lamb
 cudaError_t run_cp3(const sdad_coo3* T, const float* A, const float* B, const float* C,
                     double* loss, float* dA, float* dB, float* dC, float* dT, sdad_tmode tmode,
                     const WsLayout& L, cudaStream_t st);
+
+cudaError_t run_gnn_jvp(const sdad_csr* A, const float* H, const float* W, const float* Z,
+                        const float* valt, const float* Ht, const float* Wt, double* loss,
+                        double* loss_t, const WsLayout& L, cudaStream_t st);
 
 cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const float* Z,
                     double* loss, float* dA, float* dH, float* dW, const WsLayout& L,

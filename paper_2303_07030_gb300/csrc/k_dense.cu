@@ -1,23 +1,43 @@
-// k_dense.cu -- dense projection of the graph loss (f_in = 128, f_out = 64).
+// k_dense.cu -- dense projection of the graph loss (f_in = 128, f_out = 64),
+// on the tcgen05 tensor cores.
 //
-//   P  = H W        H: n x 128, W: 128 x 64       (tensor cores)
-//   dH = G W^T      G: n x 64                      (tensor cores)
-//   dW = H^T G      per-CTA partial sums on the CUDA cores (tiles staged by
-//                   cp.async, double-buffered), then one fixed-order reduction
+//   proj_fwd_kernel:  P  = H W                 H: n x 128, W: 128 x 64
+//   proj_bwd_kernel:  dH = G W^T  and  dW += H^T G over the CTA's rows, in one
+//                     sweep that reads each row of H and G once (per-CTA
+//                     partials of dW, then one fixed-order reduction)
 //
-// Tensor-core kernels: one CTA of 4 warps per SM, 128-row tiles.  The row
-// tile arrives by TMA in the 128-byte swizzled K-major layout; the threads
-// split it in place into TF32 hi and lo parts, and thread 0 issues
-// tcgen05.mma.kind::tf32 with the fp32 accumulator in tensor memory:
-//   D = A_hi B_hi + A_hi B_lo + A_lo B_hi      ("3xTF32": about fp32 accuracy)
-// The epilogue reads the accumulator with tcgen05.ld (warp w: TMEM lanes
-// 32w..32w+31, i.e. tile rows 32w..32w+31) and stores rows.  W (or its
-// transpose) is split and swizzled into shared memory once per CTA.
-// Waits on mbarriers are bounded (status word in the workspace header).
-#include <cudaTypedefs.h>
+// Precision: fp32 operands are split into two BF16 parts, x = hi + lo + r with
+// hi = bf16(x), lo = bf16(x - hi), |r| <= 2^-16 |x|, and each product is taken
+// as hi*hi' + hi*lo' + lo*hi' (three kind::f16 MMAs, fp32 accumulation in
+// tensor memory): about 2^-15 relative error per product, well inside the
+// 1e-4 normwise gradient tolerance (4e-6 normwise for P on the workload's
+// distributions).  BF16 parts take half the shared memory of TF32 parts, so a
+// CTA holds two tiles and W, and the MMAs issue at the BF16 rate.
+//
+// Pipeline (one CTA of 16 warps per SM, 128-row tiles t = blockIdx.x + i *
+// gridDim.x): the threads load tile i+1 into registers (16-byte streaming
+// loads) while the tensor cores work on tile i and the threads drain tile
+// i-1's accumulator from tensor memory (tcgen05.ld) to global memory.  The
+// next tile is split and written into the other of two shared-memory buffers
+// in the 128-byte swizzled layout, and thread 0 issues its MMAs; each tile's
+// MMAs commit to the mbarrier of its buffer, which frees the buffer and
+// publishes the accumulator.  Accumulators are double-buffered in tensor
+// memory.  Every wait is bounded; a kernel that gives up still waits for the
+// MMAs it issued before it frees tensor memory.
+//
+// Operand layouts (all 128-byte swizzled; a "block" is a stack of 128-byte
+// rows, each row 64 BF16 values):
+//   H tile  [2 blocks of 64 features][128 rows]  K-major A of P = H W
+//                                                (rows = M, features = K), and
+//                                                MN-major A of dW = H^T G
+//                                                (features = M, rows = K)
+//   G tile  [1 block][128 rows]                  K-major A of dH = G W^T and
+//                                                MN-major B of dW
+//   W^T     [2 blocks][64 rows = f_out]          K-major B of P
+//   W       [1 block][128 rows = f_in]           K-major B of dH
+#include <cuda_bf16.h>
 
 #include <algorithm>
-#include <mutex>
 
 #include "common.cuh"
 #include "internal.h"
@@ -27,267 +47,347 @@ namespace sdad {
 
 constexpr int kFin = 128, kFout = 64;
 constexpr int kTileM = 128;
-constexpr int kTcThreads = 128;
+constexpr int kDenseThreads = 512;
+constexpr uint32_t kBlk = 128 * 128;   // bytes of a 128-row block
 
-// ---------------------------------------------------------------------------
-// tensor maps (driver entry point obtained through the runtime)
-// ---------------------------------------------------------------------------
-namespace {
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void* p = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
-                                         &q) == cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-  });
-  return fn;
+// shared-memory map of proj_fwd_kernel (from a 1024-byte aligned base)
+constexpr uint32_t kFwdA = 0;                          // [buf][hi|lo][kb] x kBlk
+constexpr uint32_t kFwdW = kFwdA + 8 * kBlk;           // W^T: [hi|lo][kb] x 64 rows x 128 B
+constexpr uint32_t kFwdBar = kFwdW + 4 * 64 * 128;
+constexpr uint32_t kFwdSmem = kFwdBar + 32 + 1024;     // two barriers, the TMEM slot, alignment
+// shared-memory map of proj_bwd_kernel
+constexpr uint32_t kBwdG = 0;                          // [buf][hi|lo] x kBlk
+constexpr uint32_t kBwdH = kBwdG + 4 * kBlk;           // [buf][hi|lo][block] x kBlk
+constexpr uint32_t kBwdW = kBwdH + 8 * kBlk;           // W: [hi|lo] x kBlk
+constexpr uint32_t kBwdBar = kBwdW + 2 * kBlk;
+constexpr uint32_t kBwdSmem = kBwdBar + 32 + 1024;
+static_assert(kBwdSmem <= 227 * 1024, "shared memory of one CTA");
+
+__device__ __forceinline__ uint32_t bf2_bits(__nv_bfloat162 v) {
+  return *reinterpret_cast<const uint32_t*>(&v);
 }
 
-// Row-major fp32 matrix [rows x cols] read in boxes of 32 columns x 128 rows
-// with the 128-byte swizzle (rows past the end read as zero).
-bool make_map(CUtensorMap* map, const float* base, int rows, int cols) {
-  auto fn = encode_fn();
-  if (!fn) return false;
-  const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-  const cuuint64_t strides[1] = {(cuuint64_t)cols * sizeof(float)};
-  const cuuint32_t box[2] = {32, kTileM};
-  const cuuint32_t estr[2] = {1, 1};
-  return fn(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(base), dims, strides,
-            box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
-         CUDA_SUCCESS;
-}
-}  // namespace
-
-// ---------------------------------------------------------------------------
-// shared memory of the tensor-core kernels
-// ---------------------------------------------------------------------------
-// KA k-blocks (32 fp32 wide) of the A tile (128 rows) and of operand B (NB
-// rows), hi and lo copies of both, each k-block 1024-byte aligned.
-template <int KA, int NB>
-struct TcSmem {
-  float a_hi[KA][kTileM * 32];
-  float a_lo[KA][kTileM * 32];
-  float b_hi[KA][NB * 32];
-  float b_lo[KA][NB * 32];
-  uint64_t bar_load;
-  uint64_t bar_mma;
-  uint32_t tmem_base;
-};
-
-template <int KA, int NB>
-constexpr size_t tc_smem_bytes() {
-  return sizeof(TcSmem<KA, NB>) + 1024;   // room to align the base to 1024 bytes
+// hi and lo BF16 parts of four fp32 values (in order), four values per uint2
+__device__ __forceinline__ void split4(float4 x, uint2& hi, uint2& lo) {
+  const __nv_bfloat162 h01 = __floats2bfloat162_rn(x.x, x.y);
+  const __nv_bfloat162 h23 = __floats2bfloat162_rn(x.z, x.w);
+  const float2 f01 = __bfloat1622float2(h01), f23 = __bfloat1622float2(h23);
+  hi = make_uint2(bf2_bits(h01), bf2_bits(h23));
+  lo = make_uint2(bf2_bits(__floats2bfloat162_rn(x.x - f01.x, x.y - f01.y)),
+                  bf2_bits(__floats2bfloat162_rn(x.z - f23.x, x.w - f23.y)));
 }
 
-__device__ __forceinline__ unsigned char* align1024(unsigned char* p) {
-  const uint32_t a = smem_u32(p);
-  return p + ((1024u - (a & 1023u)) & 1023u);
+__device__ __forceinline__ void sts64(uint32_t addr, uint2 v) {
+  asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(addr), "r"(v.x), "r"(v.y) : "memory");
+}
+__device__ __forceinline__ void sts16(uint32_t addr, uint16_t v) {
+  asm volatile("st.shared.b16 [%0], %1;" ::"r"(addr), "h"(v) : "memory");
 }
 
-// Writes operand B (NB rows x KA*32 columns, K-major, swizzled) split into hi
-// and lo.  get(n, k) returns the fp32 value of row n, column k.
-template <int KA, int NB, class Get>
-__device__ __forceinline__ void stage_b(TcSmem<KA, NB>& S, Get get) {
-  for (int idx = threadIdx.x; idx < NB * KA * 32; idx += blockDim.x) {
-    const int nn = idx / (KA * 32), k = idx % (KA * 32);
-    const float v = get(nn, k);
-    const float hi = tc::tf32_hi(v);
-    const uint32_t off = tc::sw128_offset(nn, k & 31) / 4;
-    S.b_hi[k >> 5][off] = hi;
-    S.b_lo[k >> 5][off] = v - hi;
+// writes the hi and lo parts of one fp32 value at byte offset `off` of the
+// hi and lo copies
+__device__ __forceinline__ void put1(uint32_t hi_base, uint32_t lo_base, uint32_t off, float v) {
+  const __nv_bfloat16 h = __float2bfloat16_rn(v);
+  const __nv_bfloat16 l = __float2bfloat16_rn(v - __bfloat162float(h));
+  sts16(hi_base + off, *reinterpret_cast<const uint16_t*>(&h));
+  sts16(lo_base + off, *reinterpret_cast<const uint16_t*>(&l));
+}
+
+__device__ __forceinline__ uint32_t align1024(uint32_t a) { return (a + 1023u) & ~1023u; }
+
+// 16-byte loads of one 128-row tile of a row-major [n x (C4 * 4)] fp32 matrix
+// (rows past n read as zero): element j of this thread is float4 q = tid +
+// kDenseThreads * j, at row q / C4, column 4 (q % C4).
+template <int C4, int NJ>
+__device__ __forceinline__ void load_tile(float4 (&R)[NJ], const float* __restrict__ X, int row0,
+                                          int n) {
+#pragma unroll
+  for (int j = 0; j < NJ; ++j) {
+    const int q = threadIdx.x + kDenseThreads * j;
+    const int r = row0 + q / C4;
+    R[j] = r < n ? __ldcs(reinterpret_cast<const float4*>(X + (size_t)r * (C4 * 4)) + (q % C4))
+                 : make_float4(0.f, 0.f, 0.f, 0.f);
   }
 }
 
-// One CTA per SM; each CTA takes the 128-row tiles t = blockIdx.x, +gridDim.x.
-// X: [n x KA*32] (read through `map`), B staged from W, out: [n x NB].
-//   W_ROWS_ARE_B: operand B row n' is W row n' (dH = G W^T);
-//   otherwise operand B row n' is W column n' (P = H W).
-template <int KA, int NB, bool W_ROWS_ARE_B>
-__global__ void __launch_bounds__(kTcThreads, 1)
-    proj_tc_kernel(const __grid_constant__ CUtensorMap map, const float* __restrict__ W,
-                   float* __restrict__ out, int n, WsHeader* hdr) {
-  extern __shared__ unsigned char raw[];
-  TcSmem<KA, NB>& S = *reinterpret_cast<TcSmem<KA, NB>*>(align1024(raw));
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  constexpr uint32_t kTileBytes = KA * kTileM * 32 * sizeof(float);
-  constexpr uint32_t idesc = tc::idesc_tf32(kTileM, NB);
+// ... and their hi / lo parts into the swizzled blocks at hi_base / lo_base
+// (block b holds columns 64 b .. 64 b + 63; blocks kBlk bytes apart)
+template <int C4, int NJ>
+__device__ __forceinline__ void store_tile(const float4 (&R)[NJ], uint32_t hi_base,
+                                           uint32_t lo_base) {
+#pragma unroll
+  for (int j = 0; j < NJ; ++j) {
+    const int q = threadIdx.x + kDenseThreads * j;
+    const int r = q / C4, f = 4 * (q % C4);
+    const uint32_t off = (uint32_t)(f >> 6) * kBlk + tc::sw128_offset_b16(r, f & 63);
+    uint2 hi, lo;
+    split4(R[j], hi, lo);
+    sts64(hi_base + off, hi);
+    sts64(lo_base + off, lo);
+  }
+}
 
-  if (threadIdx.x == 0) {
-    mbar_init(&S.bar_load, 1);
-    mbar_init(&S.bar_mma, 1);
+// K-major operand descriptor of k-step s (16 BF16 = 32 bytes) in a block
+__device__ __forceinline__ uint64_t kdesc(uint32_t block, int s) {
+  return tc::smem_desc_sw128(block + 32u * (uint32_t)s);
+}
+// MN-major operand descriptor of k-step s (16 rows = 2048 bytes); MN blocks kBlk apart
+__device__ __forceinline__ uint64_t mndesc(uint32_t block, int s) {
+  return tc::smem_desc_sw128_mn(block + 2048u * (uint32_t)s, kBlk);
+}
+
+// drains COLS accumulator columns (starting at column c0 of the tile's
+// accumulator) for this warp's 32 rows into out rows of width OUTW
+template <int COLS, bool STREAM>
+__device__ __forceinline__ void drain_rows(uint32_t taddr, float* __restrict__ out, int OUTW,
+                                           int row, int col, int n) {
+  float v[COLS];
+  if constexpr (COLS == 32) tc::tmem_ld32(taddr, v);
+  else tc::tmem_ld16(taddr, v);
+  tc::tmem_wait_ld();
+  if (row < n) {
+    float4* dst = reinterpret_cast<float4*>(out + (size_t)row * OUTW + col);
+#pragma unroll
+    for (int q = 0; q < COLS / 4; ++q) {
+      const float4 w = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+      if (STREAM) __stcs(dst + q, w);
+      else dst[q] = w;
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// P = H W
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kDenseThreads, 1)
+    proj_fwd_kernel(const float* __restrict__ H, const float* __restrict__ W,
+                    float* __restrict__ P, int n, WsHeader* hdr) {
+  extern __shared__ unsigned char dense_smem[];
+  const uint32_t base = align1024(smem_u32(dense_smem));
+  unsigned char* gbase = dense_smem + (base - smem_u32(dense_smem));
+  uint64_t* bar = reinterpret_cast<uint64_t*>(gbase + kFwdBar);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + kFwdBar + 16);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  constexpr uint32_t idesc = tc::idesc_bf16(kTileM, kFout, false, false);
+  auto A = [&](int b, int part, int kb) { return base + kFwdA + (uint32_t)((b * 2 + part) * 2 + kb) * kBlk; };
+  auto Wt = [&](int part, int kb) { return base + kFwdW + (uint32_t)(part * 2 + kb) * (64 * 128); };
+
+  const int ntiles = (n + kTileM - 1) / kTileM;
+  const int grid = gridDim.x;
+  int t = blockIdx.x;
+  float4 R[8];   // the next H tile: 128 rows x 32 float4
+  if (t < ntiles) load_tile<32, 8>(R, H, t * kTileM, n);
+
+  if (tid == 0) {
+    mbar_init(&bar[0], 1);
+    mbar_init(&bar[1], 1);
     fence_mbar_init();
   }
-  if (warp == 0) tc::tmem_alloc(&S.tmem_base, NB);   // NB columns of fp32 accumulators
-  if (W_ROWS_ARE_B)
-    stage_b<KA, NB>(S, [&](int nn, int k) { return __ldg(W + (size_t)nn * (KA * 32) + k); });
-  else
-    stage_b<KA, NB>(S, [&](int nn, int k) { return __ldg(W + (size_t)k * NB + nn); });
+  if (warp == 0) tc::tmem_alloc(tmem_slot, 2 * kFout);   // two accumulators of 64 columns
+  // operand B = W^T (row n' = column n' of W), once per CTA
+  for (int idx = tid; idx < kFin * kFout; idx += kDenseThreads) {
+    const int k = idx / kFout, nn = idx % kFout;
+    const uint32_t off = tc::sw128_offset_b16(nn, k & 63);
+    put1(Wt(0, k >> 6), Wt(1, k >> 6), off, __ldg(W + idx));
+  }
   tc::fence_proxy_async_smem();
   tc::fence_before_sync();
   __syncthreads();
   tc::fence_after_sync();
-  const uint32_t tmem = S.tmem_base;
+  const uint32_t tmem = *tmem_slot;
 
-  uint32_t ph_load = 0, ph_mma = 0;
-  const int ntiles = (n + kTileM - 1) / kTileM;
-  for (int t = blockIdx.x; t < ntiles; t += gridDim.x) {
-    const int row0 = t * kTileM;
-    if (threadIdx.x == 0) {
-      mbar_arrive_expect_tx(&S.bar_load, kTileBytes);
+  const int q4 = warp & 3, cg = warp >> 2;   // epilogue: TMEM lanes 32 q4.., columns 16 cg..
+  bool ok = true;
+  int last = -1;   // local index of the last tile whose MMAs were issued
+  int i = 0;
+  for (; t < ntiles; ++i, t += grid) {
+    const int b = i & 1;
+    if (i >= 2) {   // buffer b is free once tile i-2's MMAs are done
+      ok = __syncthreads_and(mbar_wait(&bar[b], ((i >> 1) - 1) & 1, hdr));
+      if (!ok) break;
+    }
+    store_tile<32, 8>(R, A(b, 0, 0), A(b, 1, 0));
+    if (t + grid < ntiles) load_tile<32, 8>(R, H, (t + grid) * kTileM, n);
+    tc::fence_proxy_async_smem();
+    tc::fence_before_sync();
+    __syncthreads();
+    if (tid == 0) {
+      tc::fence_after_sync();
+      const uint32_t d = tmem + (uint32_t)(kFout * b);
 #pragma unroll
-      for (int kb = 0; kb < KA; ++kb) tc::tma_load_2d(S.a_hi[kb], &map, kb * 32, row0, &S.bar_load);
+      for (int kb = 0; kb < 2; ++kb)
+#pragma unroll
+        for (int s = 0; s < 4; ++s) {
+          const uint64_t ah = kdesc(A(b, 0, kb), s), al = kdesc(A(b, 1, kb), s);
+          const uint64_t bh = kdesc(Wt(0, kb), s), bl = kdesc(Wt(1, kb), s);
+          tc::mma_bf16(d, ah, bh, idesc, (kb | s) != 0);
+          tc::mma_bf16(d, ah, bl, idesc, true);
+          tc::mma_bf16(d, al, bh, idesc, true);
+        }
+      tc::mma_commit(&bar[b]);
     }
-    // all threads take the same decision (a wait that gave up ends the kernel)
-    const bool got = __syncthreads_and(mbar_wait(&S.bar_load, ph_load, hdr));
-    if (!got) {   // the tile's copy may still be landing: let it, then leave
-      mbar_drain(&S.bar_load, ph_load, hdr);
-      break;
+    last = i;
+    if (i >= 1) {   // tile i-1's accumulator to P while the tensor cores work on tile i
+      ok = __syncthreads_and(mbar_wait(&bar[b ^ 1], ((i - 1) >> 1) & 1, hdr));
+      if (!ok) break;
+      tc::fence_after_sync();
+      const int row = (t - grid) * kTileM + 32 * q4 + lane;
+      drain_rows<16, false>(tmem + ((uint32_t)(32 * q4) << 16) + (uint32_t)(kFout * (b ^ 1) + 16 * cg),
+                            P, kFout, row, 16 * cg, n);
     }
-    ph_load ^= 1;
-    // split the tile in place: hi stays, lo goes to the twin buffer
-    {
-      float4* hi4 = reinterpret_cast<float4*>(&S.a_hi[0][0]);
-      float4* lo4 = reinterpret_cast<float4*>(&S.a_lo[0][0]);
-      for (int i = threadIdx.x; i < (int)(kTileBytes / 16); i += blockDim.x) {
-        const float4 x = hi4[i];
-        const float4 h = make_float4(tc::tf32_hi(x.x), tc::tf32_hi(x.y), tc::tf32_hi(x.z),
-                                     tc::tf32_hi(x.w));
-        hi4[i] = h;
-        lo4[i] = make_float4(x.x - h.x, x.y - h.y, x.z - h.z, x.w - h.w);
-      }
+  }
+  if (ok && last >= 0) {
+    ok = __syncthreads_and(mbar_wait(&bar[last & 1], (last >> 1) & 1, hdr));
+    if (ok) {
+      tc::fence_after_sync();
+      const int row = (blockIdx.x + last * grid) * kTileM + 32 * q4 + lane;
+      drain_rows<16, false>(tmem + ((uint32_t)(32 * q4) << 16) + (uint32_t)(kFout * (last & 1) + 16 * cg),
+                            P, kFout, row, 16 * cg, n);
+    }
+  }
+  // a wait gave up: the issued MMAs still write tensor memory; let them end
+  if (!ok && last >= 0) mbar_drain(&bar[last & 1], (last >> 1) & 1, hdr);
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, 2 * kFout);
+}
+
+// ---------------------------------------------------------------------------
+// dH = G W^T and this CTA's part of dW = H^T G
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kDenseThreads, 1)
+    proj_bwd_kernel(const float* __restrict__ H, const float* __restrict__ W,
+                    const float* __restrict__ G, float* __restrict__ dH,
+                    float* __restrict__ dWpart, int n, WsHeader* hdr) {
+  extern __shared__ unsigned char dense_smem[];
+  const uint32_t base = align1024(smem_u32(dense_smem));
+  unsigned char* gbase = dense_smem + (base - smem_u32(dense_smem));
+  uint64_t* bar = reinterpret_cast<uint64_t*>(gbase + kBwdBar);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + kBwdBar + 16);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  constexpr uint32_t idesc_dh = tc::idesc_bf16(kTileM, kFin, false, false);
+  constexpr uint32_t idesc_dw = tc::idesc_bf16(kFin, kFout, true, true);
+  // dW of each tile in tensor memory (two accumulators after the two of dH);
+  // the tiles' dW are added in registers in fp32 (each thread 16 entries), so
+  // no tensor-memory accumulation runs longer than one tile's 8 k-steps
+  constexpr uint32_t kDwCol = 2 * kFin;
+  auto Gs = [&](int b, int part) { return base + kBwdG + (uint32_t)(b * 2 + part) * kBlk; };
+  auto Hs = [&](int b, int part) { return base + kBwdH + (uint32_t)((b * 2 + part) * 2) * kBlk; };
+  auto Ws = [&](int part) { return base + kBwdW + (uint32_t)part * kBlk; };
+
+  const int ntiles = (n + kTileM - 1) / kTileM;
+  const int grid = gridDim.x;
+  int t = blockIdx.x;
+  float4 RG[4], RH[8];   // the next tile: G 128 x 16 float4, H 128 x 32 float4
+  if (t < ntiles) {
+    load_tile<16, 4>(RG, G, t * kTileM, n);
+    load_tile<32, 8>(RH, H, t * kTileM, n);
+  }
+
+  if (tid == 0) {
+    mbar_init(&bar[0], 1);
+    mbar_init(&bar[1], 1);
+    fence_mbar_init();
+  }
+  if (warp == 0) tc::tmem_alloc(tmem_slot, 512);   // dH: 2 x 128 columns; dW: 2 x 64
+  // operand B of dH = W (row n' = row n' of W), once per CTA
+  for (int idx = tid; idx < kFin * kFout; idx += kDenseThreads) {
+    const int nn = idx / kFout, k = idx % kFout;
+    put1(Ws(0), Ws(1), tc::sw128_offset_b16(nn, k), __ldg(W + idx));
+  }
+  tc::fence_proxy_async_smem();
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = *tmem_slot;
+
+  const int q4 = warp & 3, cg = warp >> 2;   // epilogue: TMEM lanes 32 q4.., a quarter of the columns
+  float dwacc[16];   // this thread's entries of the CTA's dW: row 32 q4 + lane, columns 16 cg ..
+#pragma unroll
+  for (int c = 0; c < 16; ++c) dwacc[c] = 0.f;
+  // adds tile-buffer bb's dW accumulator to dwacc
+  auto add_dw = [&](int bb) {
+    float v[16];
+    tc::tmem_ld16(tmem + ((uint32_t)(32 * q4) << 16) + kDwCol + (uint32_t)(kFout * bb + 16 * cg), v);
+    tc::tmem_wait_ld();
+#pragma unroll
+    for (int c = 0; c < 16; ++c) dwacc[c] += v[c];
+  };
+  bool ok = true;
+  int last = -1;
+  int i = 0;
+  for (; t < ntiles; ++i, t += grid) {
+    const int b = i & 1;
+    if (i >= 2) {
+      ok = __syncthreads_and(mbar_wait(&bar[b], ((i >> 1) - 1) & 1, hdr));
+      if (!ok) break;
+    }
+    store_tile<16, 4>(RG, Gs(b, 0), Gs(b, 1));
+    store_tile<32, 8>(RH, Hs(b, 0), Hs(b, 1));
+    if (t + grid < ntiles) {
+      load_tile<16, 4>(RG, G, (t + grid) * kTileM, n);
+      load_tile<32, 8>(RH, H, (t + grid) * kTileM, n);
     }
     tc::fence_proxy_async_smem();
     tc::fence_before_sync();
     __syncthreads();
-    if (threadIdx.x == 0) {
+    if (tid == 0) {
       tc::fence_after_sync();
+      // dW += H^T G: M = f_in (MN-major H), N = f_out (MN-major G), K = the tile's rows
 #pragma unroll
-      for (int s = 0; s < KA * 4; ++s) {   // k-steps of 8 tf32 (32 bytes)
-        const int kb = s >> 2;
-        const uint32_t off = (uint32_t)(s & 3) * 32u;
-        const uint64_t ah = tc::smem_desc_sw128(smem_u32(S.a_hi[kb]) + off);
-        const uint64_t al = tc::smem_desc_sw128(smem_u32(S.a_lo[kb]) + off);
-        const uint64_t bh = tc::smem_desc_sw128(smem_u32(S.b_hi[kb]) + off);
-        const uint64_t bl = tc::smem_desc_sw128(smem_u32(S.b_lo[kb]) + off);
-        tc::mma_tf32(tmem, ah, bh, idesc, s > 0);
-        tc::mma_tf32(tmem, ah, bl, idesc, true);
-        tc::mma_tf32(tmem, al, bh, idesc, true);
+      for (int s = 0; s < kTileM / 16; ++s) {
+        const uint64_t ah = mndesc(Hs(b, 0), s), al = mndesc(Hs(b, 1), s);
+        const uint64_t bh = mndesc(Gs(b, 0), s), bl = mndesc(Gs(b, 1), s);
+        const uint32_t dw = tmem + kDwCol + (uint32_t)(kFout * b);
+        tc::mma_bf16(dw, ah, bh, idesc_dw, s > 0);
+        tc::mma_bf16(dw, ah, bl, idesc_dw, true);
+        tc::mma_bf16(dw, al, bh, idesc_dw, true);
       }
-      tc::mma_commit(&S.bar_mma);
-    }
-    const bool done = __syncthreads_and(mbar_wait(&S.bar_mma, ph_mma, hdr));
-    if (!done) {   // the MMAs still write tensor memory: let them end before it is freed
-      mbar_drain(&S.bar_mma, ph_mma, hdr);
-      break;
-    }
-    ph_mma ^= 1;
-    tc::fence_after_sync();
-    // epilogue: warp w owns tile rows 32w .. 32w+31 (its TMEM lane quadrant)
-    {
-      const int row = row0 + warp * 32 + lane;
-      const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16);
+      // dH = G W^T: M = rows, N = f_in, K = f_out (both K-major)
+      const uint32_t d = tmem + (uint32_t)(kFin * b);
 #pragma unroll
-      for (int c = 0; c < NB; c += 32) {
-        float v[32];
-        tc::tmem_ld32(taddr + (uint32_t)c, v);
-        tc::tmem_wait_ld();
-        if (row < n) {
-          float4* dst = reinterpret_cast<float4*>(out + (size_t)row * NB + c);
-#pragma unroll
-          for (int q = 0; q < 8; ++q)
-            dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-        }
+      for (int s = 0; s < (dH ? kFout / 16 : 0); ++s) {
+        const uint64_t ah = kdesc(Gs(b, 0), s), al = kdesc(Gs(b, 1), s);
+        const uint64_t bh = kdesc(Ws(0), s), bl = kdesc(Ws(1), s);
+        tc::mma_bf16(d, ah, bh, idesc_dh, s > 0);
+        tc::mma_bf16(d, ah, bl, idesc_dh, true);
+        tc::mma_bf16(d, al, bh, idesc_dh, true);
       }
+      tc::mma_commit(&bar[b]);
     }
-    tc::fence_before_sync();
-    __syncthreads();
+    last = i;
+    if (i >= 1) {   // tile i-1's dH to memory and its dW into dwacc
+      ok = __syncthreads_and(mbar_wait(&bar[b ^ 1], ((i - 1) >> 1) & 1, hdr));
+      if (!ok) break;
+      tc::fence_after_sync();
+      const int row = (t - grid) * kTileM + 32 * q4 + lane;
+      if (dH)
+        drain_rows<32, true>(tmem + ((uint32_t)(32 * q4) << 16) + (uint32_t)(kFin * (b ^ 1) + 32 * cg),
+                             dH, kFin, row, 32 * cg, n);
+      add_dw(b ^ 1);
+    }
   }
-  tc::fence_after_sync();
+  if (ok && last >= 0) {
+    ok = __syncthreads_and(mbar_wait(&bar[last & 1], (last >> 1) & 1, hdr));
+    if (ok) {
+      tc::fence_after_sync();
+      const int row = (blockIdx.x + last * grid) * kTileM + 32 * q4 + lane;
+      if (dH)
+        drain_rows<32, true>(tmem + ((uint32_t)(32 * q4) << 16) + (uint32_t)(kFin * (last & 1) + 32 * cg),
+                             dH, kFin, row, 32 * cg, n);
+      add_dw(last & 1);
+      // this CTA's dW: TMEM lane = f_in, column = f_out
+      float4* dst = reinterpret_cast<float4*>(dWpart + (size_t)blockIdx.x * kFin * kFout +
+                                              (size_t)(32 * q4 + lane) * kFout + 16 * cg);
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        dst[q] = make_float4(dwacc[4 * q], dwacc[4 * q + 1], dwacc[4 * q + 2], dwacc[4 * q + 3]);
+    }
+  }
+  if (!ok && last >= 0) mbar_drain(&bar[last & 1], (last >> 1) & 1, hdr);
+  tc::fence_before_sync();
   __syncthreads();
-  if (warp == 0) tc::tmem_dealloc(tmem, NB);
-}
-
-// dW partials: dWpart[b] = sum over the CTA's 64-row tiles of H_tile^T G_tile.
-// Thread (ta, tb) owns dW[4*ta .. +3][8*tb .. +7] in registers.  The tiles go
-// through two shared-memory stages filled by cp.async (16-byte copies; rows
-// past n are zero-filled), so the next tile loads while this one is used.
-constexpr int kDwRows = 64;
-struct DwStage {
-  float H[kDwRows * kFin];
-  float G[kDwRows * kFout];
-};
-
-__device__ __forceinline__ void cp_async16(void* dst, const void* src, bool valid) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_u32(dst)), "l"(src),
-               "r"(valid ? 16 : 0)
-               : "memory");
-}
-
-// Issues the copies of the tile starting at row r0 into stage S (one group).
-__device__ __forceinline__ void dw_load(DwStage& S, const float* __restrict__ H,
-                                        const float* __restrict__ G, int r0, int n) {
-  for (int i = threadIdx.x; i < kDwRows * kFin / 4; i += blockDim.x) {
-    const int rr = i / (kFin / 4);
-    const bool ok = r0 + rr < n;
-    cp_async16(S.H + 4 * i, ok ? H + (size_t)r0 * kFin + 4 * i : H, ok);
-  }
-  for (int i = threadIdx.x; i < kDwRows * kFout / 4; i += blockDim.x) {
-    const int rr = i / (kFout / 4);
-    const bool ok = r0 + rr < n;
-    cp_async16(S.G + 4 * i, ok ? G + (size_t)r0 * kFout + 4 * i : G, ok);
-  }
-  asm volatile("cp.async.commit_group;" ::: "memory");
-}
-
-__global__ void __launch_bounds__(256)
-    proj_dw_kernel(const float* __restrict__ H, const float* __restrict__ G,
-                   float* __restrict__ dWpart, int n) {
-  extern __shared__ __align__(16) unsigned char dw_raw[];
-  DwStage* st = reinterpret_cast<DwStage*>(dw_raw);   // two stages
-  const int tid = threadIdx.x, tb = tid & 7, ta = tid >> 3;   // ta 0..31, tb 0..7
-  float acc[4][8];
-#pragma unroll
-  for (int i = 0; i < 4; ++i)
-#pragma unroll
-    for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
-  const int stride = gridDim.x * kDwRows;
-  int r0 = blockIdx.x * kDwRows;
-  if (r0 < n) dw_load(st[0], H, G, r0, n);
-  for (int it = 0; r0 < n; ++it, r0 += stride) {
-    DwStage& cur = st[it & 1];
-    const bool more = r0 + stride < n;
-    if (more) dw_load(st[(it + 1) & 1], H, G, r0 + stride, n);
-    if (more)
-      asm volatile("cp.async.wait_group 1;" ::: "memory");   // this tile's group is done
-    else
-      asm volatile("cp.async.wait_group 0;" ::: "memory");
-    __syncthreads();
-#pragma unroll 4
-    for (int r = 0; r < kDwRows; ++r) {
-      const float4 h = *reinterpret_cast<const float4*>(cur.H + r * kFin + 4 * ta);
-      const float4 g0 = *reinterpret_cast<const float4*>(cur.G + r * kFout + 8 * tb);
-      const float4 g1 = *reinterpret_cast<const float4*>(cur.G + r * kFout + 8 * tb + 4);
-      const float hv[4] = {h.x, h.y, h.z, h.w};
-      const float gv[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(hv[i], gv[j], acc[i][j]);
-    }
-    __syncthreads();   // the stage is refilled two tiles on
-  }
-  float* dst = dWpart + (size_t)blockIdx.x * kFin * kFout;
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    float4* d = reinterpret_cast<float4*>(dst + (4 * ta + i) * kFout + 8 * tb);
-    d[0] = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
-    d[1] = make_float4(acc[i][4], acc[i][5], acc[i][6], acc[i][7]);
-  }
+  if (warp == 0) tc::tmem_dealloc(tmem, 512);
 }
 
 // dW[e] = sum_p parts[p][e], p in ascending order.
@@ -300,55 +400,54 @@ __global__ void dw_reduce_kernel(const float* __restrict__ parts, int nparts,
   dW[e] = s;
 }
 
-namespace {
-
-template <int KA, int NB, bool T>
-cudaError_t launch_tc(const char* name, const float* X, int xcols, const float* W, float* out,
-                      int n, WsHeader* hdr, cudaStream_t st) {
-  auto kern = proj_tc_kernel<KA, NB, T>;
-  constexpr size_t smem = tc_smem_bytes<KA, NB>();
-  cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void*>(kern), (int)smem);
-  if (e != cudaSuccess) return e;
-  if (n <= 0) return cudaSuccess;
-  CUtensorMap map;
-  if (!make_map(&map, X, n, xcols)) return cudaErrorInvalidValue;
-  const int tiles = (n + kTileM - 1) / kTileM;
-  const int grid = std::min(tiles, device_sm_count());
-  {
-    KTimer t(name, st);
-    kern<<<grid, kTcThreads, smem, st>>>(map, W, out, n, hdr);
-  }
-  return cudaGetLastError();
+__global__ void zero_dw_kernel(float* __restrict__ dW) {
+  const int e = blockIdx.x * blockDim.x + threadIdx.x;
+  if (e < kFin * kFout) dW[e] = 0.f;
 }
 
+namespace {
+int dense_grid(int n) {
+  const int tiles = (n + kTileM - 1) / kTileM;
+  return std::max(1, std::min(tiles, device_sm_count()));
+}
 }  // namespace
 
 cudaError_t dense_proj_fwd(const float* H, const float* W, float* P, int n, WsHeader* hdr,
                            cudaStream_t st) {
-  // P = H W: A = H (K = 128 -> 4 k-blocks), operand B row n' = W column n' (64 rows)
-  return launch_tc<4, kFout, false>("proj_fwd", H, kFin, W, P, n, hdr, st);
+  cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void*>(proj_fwd_kernel), (int)kFwdSmem);
+  if (e != cudaSuccess || n <= 0) return e;
+  {
+    KTimer t("proj_fwd", st);
+    proj_fwd_kernel<<<dense_grid(n), kDenseThreads, kFwdSmem, st>>>(H, W, P, n, hdr);
+  }
+  return cudaGetLastError();
 }
 
 cudaError_t dense_proj_bwd(const float* H, const float* W, const float* G, float* dH,
                            float* dWpart, float* dW, int n, WsHeader* hdr, cudaStream_t st) {
-  cudaError_t e;
-  if (dH) {
-    // dH = G W^T: A = G (K = 64 -> 2 k-blocks), operand B row n' = W row n' (128 rows)
-    if ((e = launch_tc<2, kFin, true>("proj_dh", G, kFout, W, dH, n, hdr, st)) != cudaSuccess)
-      return e;
+  // dH and dW come from one sweep (which skips dH's MMAs and stores when dH
+  // is not wanted); dW's per-CTA partials are summed afterwards
+  cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void*>(proj_bwd_kernel), (int)kBwdSmem);
+  if (e != cudaSuccess) return e;
+  if (n <= 0) {
+    if (dW) {
+      zero_dw_kernel<<<(kFin * kFout + 255) / 256, 256, 0, st>>>(dW);
+      return cudaGetLastError();
+    }
+    return cudaSuccess;
   }
-  if (!dW) return cudaSuccess;
+  const int grid = dense_grid(n);
+  static_assert(kDwParts >= 152, "one dW partial per CTA");
+  if (grid > kDwParts) return cudaErrorInvalidConfiguration;
   {
-    e = ensure_dynamic_smem(reinterpret_cast<const void*>(proj_dw_kernel),
-                            (int)(2 * sizeof(DwStage)));
-    if (e != cudaSuccess) return e;
-    KTimer t("proj_dw", st);
-    proj_dw_kernel<<<kDwParts, 256, 2 * sizeof(DwStage), st>>>(H, G, dWpart, n);
+    KTimer t("proj_bwd", st);
+    proj_bwd_kernel<<<grid, kDenseThreads, kBwdSmem, st>>>(H, W, G, dH, dWpart, n, hdr);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if (!dW) return cudaSuccess;
   {
     KTimer t("dw_reduce", st);
-    dw_reduce_kernel<<<(kFin * kFout + 255) / 256, 256, 0, st>>>(dWpart, kDwParts, dW);
+    dw_reduce_kernel<<<(kFin * kFout + 255) / 256, 256, 0, st>>>(dWpart, grid, dW);
   }
   return cudaGetLastError();
 }

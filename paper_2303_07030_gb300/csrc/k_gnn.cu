@@ -16,13 +16,20 @@
 //      a 4-byte store per key instead of a second 256-byte gather of P
 //   6. fix of the cut columns
 //   7. dH = G W^T and dW = H^T G                          (dense projection)
-// Lane layout of the walks: a warp takes one key at a time; lane l holds the
-// elements 2l, 2l+1 of the 64-wide rows (one 256-byte coalesced gather per
-// key); eight gathers are issued before they are used.  Every sum has a fixed
-// order (chunk structure, lane layout), so the results are reproducible.
+//
+// Lane layout of the walks: a warp takes two keys at a time, one per half
+// warp; lane l of half h = l / 16 holds elements 4(l % 16) .. 4(l % 16) + 3
+// of the 64-wide rows, so one warp instruction gathers two 256-byte rows with
+// 16-byte loads.  Sixteen keys (eight pairs) are gathered before they are
+// used.  Each half keeps its own partial sum of the open segment; a segment
+// that ends is closed by adding the two halves (one shuffle of a float4), so
+// every sum has a fixed order (chunk structure, lane layout) and the results
+// are reproducible.
 #include <algorithm>
+#include <climits>
 
 #include "common.cuh"
+#include "halfwarp.cuh"
 #include "internal.h"
 
 namespace sdad {
@@ -30,9 +37,7 @@ namespace sdad {
 constexpr int kWideChunk = kMinCap;   // 1024 keys: the piece slots are per kMinCap keys
 constexpr int kWideThreads = 256;
 constexpr int kWideWarps = kWideThreads / 32;
-constexpr int kWideBatch = 8;         // gathers in flight per warp
-constexpr int kColPrefetchP = 2;      // column walk with dA: next columns' P rows prefetched into L2
-constexpr bool kFwdPrefetchZ = false;  // forward walk: a row's Z prefetched into L2 when it begins (measured slower)
+constexpr int kWalkCtas = 3;          // resident CTAs per SM the walks are compiled for (<= 85 registers)
 
 __device__ __forceinline__ float2 ld2(const float* base, int r, int lane) {
   return __ldg(reinterpret_cast<const float2*>(base + (size_t)r * 64) + lane);
@@ -40,128 +45,154 @@ __device__ __forceinline__ float2 ld2(const float* base, int r, int lane) {
 __device__ __forceinline__ void st2(float* base, int r, int lane, float2 v) {
   reinterpret_cast<float2*>(base + (size_t)r * 64)[lane] = v;
 }
-__device__ __forceinline__ float wsum(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(FULL_MASK, v, o);
-  return v;
-}
 
-// One chunk of a compressed structure (ptr, idx, val), walked key by key:
-// calls vis.segment(s, acc, ...) for every segment whose keys in the chunk
-// are done (acc = sum of val * X[idx] over them, 64-wide, lane layout above).
-// Segments without keys are skipped (gnn_empty_kernel handles them).
-template <class Vis>
-__device__ __forceinline__ void wide_walk(const int32_t* __restrict__ ptr, int nseg,
-                                          const int32_t* __restrict__ idx,
-                                          const float* __restrict__ val,
-                                          const float* __restrict__ X, int nnz, int cs, int ce,
-                                          int hint, int lane, Vis& vis, int* seg_out) {
-  // the segment holding key cs: the last s with ptr[s] <= cs
-  int s = warp_gallop_lower_bound(ptr, hint, nseg + 1, cs + 1) - 1;
-  int s0 = __ldg(ptr + s), s1 = __ldg(ptr + s + 1);
-  vis.begin(s);
-  float2 acc = make_float2(0.f, 0.f);
-  for (int base = cs; base < ce; base += 32) {
-    const int nk = min(32, ce - base);
-    const int jl = lane < nk ? __ldg(idx + base + lane) : 0;
-    const float al = lane < nk ? __ldg(val + base + lane) : 0.f;
-    for (int k0 = 0; k0 < nk; k0 += kWideBatch) {
-      float2 x[kWideBatch];
-#pragma unroll
-      for (int u = 0; u < kWideBatch; ++u) {
-        const int j = __shfl_sync(FULL_MASK, jl, (k0 + u) & 31);
-        x[u] = (k0 + u < nk) ? ld2(X, j, lane) : make_float2(0.f, 0.f);
-      }
-#pragma unroll
-      for (int u = 0; u < kWideBatch; ++u) {
-        const float a = __shfl_sync(FULL_MASK, al, (k0 + u) & 31);
-        if (k0 + u >= nk) break;   // warp-uniform
-        const int p = base + k0 + u;
-        if (p >= s1) {   // segment s is done: report it, move to the segment of p
-          vis.segment(s, s0, s1, acc, cs, ce);
-          s = warp_gallop_lower_bound(ptr, s + 1, nseg + 1, p + 1) - 1;
-          s0 = __ldg(ptr + s);
-          s1 = __ldg(ptr + s + 1);
-          vis.begin(s);
-          acc = make_float2(0.f, 0.f);
-        }
-        acc.x = fmaf(a, x[u].x, acc.x);
-        acc.y = fmaf(a, x[u].y, acc.y);
-      }
-    }
+// The segment holding key p, searched from segment `lo` on (ptr[lo] <= p):
+// the last s with ptr[s] <= p, with its bounds.  The next 32 pointers are
+// read in one coalesced load and the bounds taken from it by shuffles;
+// beyond them, a binary search.  Called by the whole warp.
+struct Seg {
+  int s, s0, s1;
+};
+__device__ __forceinline__ Seg next_segment(const int32_t* __restrict__ ptr, int nseg, int lo,
+                                            int p, int lane) {
+  // first i in [lo + 1, nseg] with ptr[i] > p; the segment is i - 1
+  const int i = lo + 1 + lane;
+  const int pv = i <= nseg ? __ldg(ptr + i) : INT_MAX;
+  const unsigned b = __ballot_sync(FULL_MASK, pv > p);
+  if (b) {
+    const int f = __ffs(b) - 1;
+    const int s1 = __shfl_sync(FULL_MASK, pv, f);
+    const int before = __shfl_sync(FULL_MASK, pv, (f + 31) & 31);
+    // f = 0 would mean p lies in segment lo itself (not so where the walks call this)
+    return Seg{lo + f, f ? before : __ldg(ptr + lo), s1};
   }
-  vis.segment(s, s0, s1, acc, cs, ce);
-  *seg_out = s;
-}
-
-// Sums eight values over the warp: on return lane l holds the sum of value
-// (l >> 2) & 7 (a butterfly that halves the values at each of the first three
-// steps: 9 shuffles for 8 sums).
-__device__ __forceinline__ float reduce8(float (&t)[kWideBatch], int lane) {
-  static_assert(kWideBatch == 8, "eight values");
-  const bool b4 = lane & 16, b3 = lane & 8, b2 = lane & 4;
-  float u[4];
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {   // keep values 4*b4 + i, send the other half
-    const float keep = b4 ? t[i + 4] : t[i], send = b4 ? t[i] : t[i + 4];
-    u[i] = keep + __shfl_xor_sync(FULL_MASK, send, 16);
-  }
-  float w[2];
-#pragma unroll
-  for (int i = 0; i < 2; ++i) {   // keep 2*b3 + i of u
-    const float keep = b3 ? u[i + 2] : u[i], send = b3 ? u[i] : u[i + 2];
-    w[i] = keep + __shfl_xor_sync(FULL_MASK, send, 8);
-  }
-  const float keep = b2 ? w[1] : w[0], send = b2 ? w[0] : w[1];
-  float x = keep + __shfl_xor_sync(FULL_MASK, send, 4);
-  x += __shfl_xor_sync(FULL_MASK, x, 2);
-  x += __shfl_xor_sync(FULL_MASK, x, 1);
-  return x;   // value index 4*b4 + 2*b3 + b2 = (lane >> 2) & 7
-}
-
-// dA[p] = d . P[colidx[p]] for p in [q0, q1): eight gathers in flight, the
-// eight dot products reduced together, 32 results stored together.
-__device__ __forceinline__ void sddmm_range(const int32_t* __restrict__ colidx,
-                                            const float* __restrict__ P, float2 d,
-                                            float* __restrict__ dA, int q0, int q1, int lane) {
-  for (int base = q0; base < q1; base += 32) {
-    const int nk = min(32, q1 - base);
-    const int jl = lane < nk ? __ldg(colidx + base + lane) : 0;
-    float mine = 0.f;
-    for (int k0 = 0; k0 < nk; k0 += kWideBatch) {
-      float t[kWideBatch];
-#pragma unroll
-      for (int u = 0; u < kWideBatch; ++u) {
-        const int j = __shfl_sync(FULL_MASK, jl, (k0 + u) & 31);
-        const float2 x = (k0 + u < nk) ? ld2(P, j, lane) : make_float2(0.f, 0.f);
-        t[u] = fmaf(d.y, x.y, d.x * x.x);
-      }
-      const float r = reduce8(t, lane);
-      // key k0 + ((lane >> 2) & 7) is held by lanes 4 * k .. 4 * k + 3
-      const float got = __shfl_sync(FULL_MASK, r, ((lane - k0) & 7) * 4);
-      if (lane >= k0 && lane < k0 + kWideBatch) mine = got;
-    }
-    if (lane < nk) dA[base + lane] = mine;
-  }
+  const int s = warp_lower_bound(ptr, lo + 33, nseg + 1, p + 1) - 1;
+  return Seg{s, __ldg(ptr + s), __ldg(ptr + s + 1)};
 }
 
 struct ChunkPieces {
   float* __restrict__ pfirst;   // [chunks x 64]: part of a segment begun in an earlier chunk
   float* __restrict__ plast;    // [chunks x 64]: part of the segment that continues past it
   int* __restrict__ lastseg;    // that segment, or -1
-  // stores the chunk's part of a cut segment; returns true for a cut one
-  __device__ __forceinline__ bool cut(int ch, int s, int s0, int s1, int cs, int ce, float2 acc,
+  // stores the chunk's part of a cut segment (half 0 of the warp writes the
+  // row); returns true for a cut one
+  __device__ __forceinline__ bool cut(int ch, int s, int s0, int s1, int cs, int ce, float4 tot,
                                       int lane) const {
     if (s0 >= cs && s1 <= ce) return false;
-    if (s0 < cs) {
-      st2(pfirst, ch, lane, acc);
-    } else {
-      st2(plast, ch, lane, acc);
-      if (lane == 0) lastseg[ch] = s;
+    if (lane < 16) {
+      if (s0 < cs) {
+        st4(pfirst, ch, lane, tot);
+      } else {
+        st4(plast, ch, lane, tot);
+        if (lane == 0) lastseg[ch] = s;
+      }
     }
     return true;
   }
 };
+
+// One chunk [cs, ce) of a compressed structure (ptr, idx, val), walked two
+// keys at a time: calls vis.segment(s, s0, s1, tot, cs, ce) for every segment
+// whose keys in the chunk are done (tot = sum of val * X[idx] over them,
+// 64-wide, float4 per lane, both halves holding the whole row), and
+// vis.key(h, x, q) for every key q (x = the gathered row, held by half h) at
+// the moment the walk is in q's segment.  Segments without keys are skipped
+// (gnn_empty_kernel handles them).
+template <class Vis>
+__device__ __forceinline__ void pair_walk(const int32_t* __restrict__ ptr, int nseg,
+                                          const int32_t* __restrict__ idx,
+                                          const float* __restrict__ val,
+                                          const float* __restrict__ X, int cs, int ce, int hint,
+                                          int lane, Vis& vis, int* seg_out) {
+  const int h = lane >> 4, sl = lane & 15;
+  // the segment holding key cs: the last s with ptr[s] <= cs
+  int s = warp_gallop_lower_bound(ptr, hint, nseg + 1, cs + 1) - 1;
+  int s0 = __ldg(ptr + s), s1 = __ldg(ptr + s + 1);
+  vis.begin(s, lane);
+  float4 acc = zero4();
+  for (int base = cs; base < ce; base += 32) {
+    const int nk = min(32, ce - base);
+    const int jl = lane < nk ? __ldg(idx + base + lane) : 0;
+    const float al = lane < nk ? __ldg(val + base + lane) : 0.f;
+    vis.window(base, nk, lane);
+    for (int k0 = 0; k0 < nk; k0 += 2 * kPairs) {
+      float4 x[kPairs];
+#pragma unroll
+      for (int u = 0; u < kPairs; ++u) {
+        const int kk = k0 + 2 * u + h;
+        const int j = __shfl_sync(FULL_MASK, jl, kk & 31);
+        x[u] = kk < nk ? ld4(X, j, sl) : zero4();
+      }
+#pragma unroll
+      for (int u = 0; u < kPairs; ++u) {
+        const int kk = k0 + 2 * u;   // this pair: keys kk (half 0) and kk + 1 (half 1)
+        const float a = __shfl_sync(FULL_MASK, al, (kk + h) & 31);
+        if (kk >= nk) break;   // warp-uniform
+        const int p0 = base + kk;
+        const bool two = kk + 1 < nk;
+        if ((two ? p0 + 1 : p0) < s1) {   // both keys in segment s (the usual case)
+          acc = fma4(a, x[u], acc);        // an absent second key adds a zero row
+          vis.key(h, x[u], kk + h, u);
+          continue;
+        }
+        // a segment ends inside the pair
+        if (p0 >= s1) {
+          vis.segment(s, s0, s1, join_halves(acc), cs, ce);
+          const Seg g = next_segment(ptr, nseg, s, p0, lane);
+          s = g.s; s0 = g.s0; s1 = g.s1;
+          vis.begin(s, lane);
+          acc = zero4();
+        }
+        if (h == 0) acc = fma4(a, x[u], acc);
+        vis.key_if(h == 0, x[u], kk, u);
+        if (two) {
+          if (p0 + 1 >= s1) {
+            vis.segment(s, s0, s1, join_halves(acc), cs, ce);
+            const Seg g = next_segment(ptr, nseg, s, p0 + 1, lane);
+            s = g.s; s0 = g.s0; s1 = g.s1;
+            vis.begin(s, lane);
+            acc = zero4();
+          }
+          if (h == 1) acc = fma4(a, x[u], acc);
+          vis.key_if(h == 1, x[u], kk + 1, u);
+        }
+      }
+      vis.batch_done(k0, nk, lane);
+    }
+  }
+  vis.segment(s, s0, s1, join_halves(acc), cs, ce);
+  *seg_out = s;
+}
+
+
+
+// dA[p] = d . P[colidx[p]] for p in [q0, q1): sixteen gathers in flight, the
+// sixteen dot products reduced together, 32 results stored together.  d is
+// the row's float4 of this lane's elements (the same in both halves).
+__device__ __forceinline__ void sddmm_range(const int32_t* __restrict__ colidx,
+                                            const float* __restrict__ P, float4 d,
+                                            float* __restrict__ dA, int q0, int q1, int lane) {
+  const int h = lane >> 4, sl = lane & 15;
+  for (int base = q0; base < q1; base += 32) {
+    const int nk = min(32, q1 - base);
+    const int jl = lane < nk ? __ldg(colidx + base + lane) : 0;
+    float mine = 0.f;
+    for (int k0 = 0; k0 < nk; k0 += 2 * kPairs) {
+      float t[kPairs];
+#pragma unroll
+      for (int u = 0; u < kPairs; ++u) {
+        const int kk = k0 + 2 * u + h;
+        const int j = __shfl_sync(FULL_MASK, jl, kk & 31);
+        const float4 x = kk < nk ? ld4(P, j, sl) : zero4();
+        t[u] = dot4(d, x);
+      }
+      const float r = reduce_half8(t, lane);
+      const float got = __shfl_sync(FULL_MASK, r, batch_src_lane((lane - k0) & 15));
+      if (lane >= k0 && lane < k0 + 2 * kPairs) mine = got;
+    }
+    if (lane < nk) dA[base + lane] = mine;
+  }
+}
 
 // ---- 2: forward walk -------------------------------------------------------
 struct FwdVisit {
@@ -174,21 +205,29 @@ struct FwdVisit {
   int ch, lane;
   double loss;   // this lane's part
 
-  // row r begins: its row of Z (read when the row is done) into L2 now
-  __device__ __forceinline__ void begin(int r) {
-    if (kFwdPrefetchZ && lane == 0) prefetch_l2_range(Z, (long long)r * 64, (long long)(r + 1) * 64);
-  }
-  __device__ __forceinline__ void segment(int r, int s0, int s1, float2 acc, int cs, int ce) {
-    if (pc.cut(ch, r, s0, s1, cs, ce, acc, lane)) return;
-    const float2 z = ld2(Z, r, lane);
-    const float2 d = make_float2(acc.x - z.x, acc.y - z.y);
-    st2(D, r, lane, d);
-    loss += 0.5 * (double)fmaf(d.x, d.x, d.y * d.y);
+  __device__ __forceinline__ void begin(int, int) {}
+  __device__ __forceinline__ void window(int, int, int) {}
+  __device__ __forceinline__ void key(int, float4, int, int) {}
+  __device__ __forceinline__ void key_if(bool, float4, int, int) {}
+  __device__ __forceinline__ void batch_done(int, int, int) {}
+  __device__ __forceinline__ void segment(int r, int s0, int s1, float4 tot, int cs, int ce) {
+    if (pc.cut(ch, r, s0, s1, cs, ce, tot, lane)) return;
+    const int sl = lane & 15;
+    const float4 z = ld4(Z, r, sl);
+    const float4 d = make_float4(tot.x - z.x, tot.y - z.y, tot.z - z.z, tot.w - z.w);
+    if (lane < 16) {
+      st4(D, r, sl, d);
+      loss += 0.5 * (double)dot4(d, d);
+    }
     if (dA) sddmm_range(colidx, P, d, dA, s0, s1, lane);
   }
 };
 
-__global__ void __launch_bounds__(kWideThreads)
+// WITH_DA: dA of the rows finished inside a chunk (when no transpose
+// permutation lets the column walk compute it); a template parameter so that
+// the plain walk does not carry the SDDMM's registers.
+template <bool WITH_DA>
+__global__ void __launch_bounds__(kWideThreads, kWalkCtas)
     gnn_fwd_kernel(const int32_t* __restrict__ rowptr, const int32_t* __restrict__ colidx,
                    const float* __restrict__ val, int m, int nnz, int nchunks,
                    const float* __restrict__ P, const float* __restrict__ Z, float* __restrict__ D,
@@ -198,14 +237,14 @@ __global__ void __launch_bounds__(kWideThreads)
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int gw = blockIdx.x * kWideWarps + warp, nw = gridDim.x * kWideWarps;
   const int c0 = (int)(((long long)nchunks * gw) / nw), c1 = (int)(((long long)nchunks * (gw + 1)) / nw);
-  FwdVisit vis{colidx, P, Z, D, dA, pc, 0, lane, 0.0};
+  FwdVisit vis{colidx, P, Z, D, WITH_DA ? dA : nullptr, pc, 0, lane, 0.0};
   int hint = 0;
   for (int ch = c0; ch < c1; ++ch) {
     const int cs = ch * kWideChunk, ce = min(cs + kWideChunk, nnz);
     if (lane == 0) pc.lastseg[ch] = -1;
     __syncwarp();
     vis.ch = ch;
-    if (cs < ce) wide_walk(rowptr, m, colidx, val, P, nnz, cs, ce, hint, lane, vis, &hint);
+    if (cs < ce) pair_walk(rowptr, m, colidx, val, P, cs, ce, hint, lane, vis, &hint);
   }
   const double cta = block_sum_d(vis.loss, red);
   publish_loss(cta, hdr, partials, 0, false, 1.0, loss_out, red);
@@ -317,7 +356,7 @@ __global__ void __launch_bounds__(kWideThreads)
     gnn_cut_sddmm_kernel(const int32_t* __restrict__ rowptr, const int32_t* __restrict__ colidx,
                          int m, int nnz, int nchunks, const float* __restrict__ P,
                          const float* __restrict__ D, float* __restrict__ dA) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, sl = lane & 15;
   const int gw = blockIdx.x * kWideWarps + warp, nw = gridDim.x * kWideWarps;
   for (int ch = gw; ch < nchunks; ch += nw) {
     const int cs = ch * kWideChunk, ce = min(cs + kWideChunk, nnz);
@@ -326,91 +365,67 @@ __global__ void __launch_bounds__(kWideThreads)
     const int rl = warp_lower_bound(rowptr, rf, m + 1, ce) - 1;          // row of key ce - 1
     const int f0 = __ldg(rowptr + rf), f1 = __ldg(rowptr + rf + 1);
     if (f0 < cs || f1 > ce)   // the first row is cut
-      sddmm_range(colidx, P, ld2(D, rf, lane), dA, cs, min(f1, ce), lane);
+      sddmm_range(colidx, P, ld4(D, rf, sl), dA, cs, min(f1, ce), lane);
     if (rl != rf) {
       const int l1 = __ldg(rowptr + rl + 1);
       if (l1 > ce)   // the last row continues past the chunk
-        sddmm_range(colidx, P, ld2(D, rl, lane), dA, __ldg(rowptr + rl), ce, lane);
+        sddmm_range(colidx, P, ld4(D, rl, sl), dA, __ldg(rowptr + rl), ce, lane);
     }
   }
 }
 
 // ---- 5: G = A^T D over the CSC twin ------------------------------------------
+// Visitor of the column walk.  With `perm` (the CSC twin's transpose
+// permutation) it also computes, for each key q of column c (row i),
+// dA[perm[q]] = D_i . P_c, with P_c held by the lanes while the walk is in
+// column c -- the D row is the one gathered for G, so dA costs no gather.
+// Sixteen dot products are reduced together (reduce_half8).
 struct ColVisit {
   float* __restrict__ G;
   ChunkPieces pc;
-  int ch, lane;
-  __device__ __forceinline__ void begin(int) {}
-  __device__ __forceinline__ void segment(int c, int s0, int s1, float2 acc, int cs, int ce) {
-    if (pc.cut(ch, c, s0, s1, cs, ce, acc, lane)) return;
-    st2(G, c, lane, acc);
+  const int32_t* __restrict__ perm;   // NULL: no dA
+  const float* __restrict__ P;
+  float* __restrict__ dA;
+  int n, ch, lane;
+  int ql;            // perm of this lane's key of the current 32-key window
+  float4 pcol;       // P row of the current column (this lane's elements)
+  float t[kPairs];   // this lane's parts of the batch's dot products
+
+  __device__ __forceinline__ void begin(int c, int lane_) {
+    if (!perm) return;
+    pcol = ld4(P, c, lane_ & 15);
+    // the next columns' rows of P into L2 (they are loaded at the next switches)
+    if (lane_ < 2 && c + 1 + lane_ < n)
+      prefetch_l2_range(P, (long long)(c + 1 + lane_) * 64, (long long)(c + 2 + lane_) * 64);
+  }
+  __device__ __forceinline__ void window(int base, int nk, int lane_) {
+    if (perm) ql = lane_ < nk ? __ldg(perm + base + lane_) : 0;
+  }
+  __device__ __forceinline__ void key(int, float4 x, int, int u) {
+    if (perm) t[u] = dot4(x, pcol);
+  }
+  __device__ __forceinline__ void key_if(bool mine, float4 x, int, int u) {
+    if (perm && mine) t[u] = dot4(x, pcol);
+  }
+  __device__ __forceinline__ void batch_done(int k0, int nk, int lane_) {
+    if (!perm) return;
+    const float r = reduce_half8(t, lane_);
+    // lane (h, sl) with sl even holds key k0 + 2 ((sl >> 1) & 7) + h
+    const int sl = lane_ & 15;
+    const int kk = k0 + 2 * ((sl >> 1) & 7) + (lane_ >> 4);
+    const int q = __shfl_sync(FULL_MASK, ql, kk & 31);
+    if ((sl & 1) == 0 && kk < nk) dA[q] = r;
+#pragma unroll
+    for (int u = 0; u < kPairs; ++u) t[u] = 0.f;
+  }
+  __device__ __forceinline__ void segment(int c, int s0, int s1, float4 tot, int cs, int ce) {
+    if (pc.cut(ch, c, s0, s1, cs, ce, tot, lane)) return;
+    if (lane < 16) st4(G, c, lane, tot);
   }
 };
 
-// The column walk with the gradient on the keys: as wide_walk over the CSC
-// twin (gathering D rows), and for each key q of column c (row i) also
-// dA[perm[q]] = D_i . P_c, with P_c held by the lanes while the walk is in
-// column c -- the D row is the one gathered for G, so dA costs no gather.
-// Eight dot products are reduced together (reduce8); lane 4k stores key k's.
-__device__ __forceinline__ void col_walk_sddmm(const int32_t* __restrict__ colptr, int n,
-                                               const int32_t* __restrict__ rowidx,
-                                               const float* __restrict__ val_csc,
-                                               const int32_t* __restrict__ perm,
-                                               const float* __restrict__ D,
-                                               const float* __restrict__ P,
-                                               float* __restrict__ dA, int cs, int ce, int hint,
-                                               int lane, ColVisit& vis, int* seg_out) {
-  int s = warp_gallop_lower_bound(colptr, hint, n + 1, cs + 1) - 1;
-  int s0 = __ldg(colptr + s), s1 = __ldg(colptr + s + 1);
-  float2 pcol = ld2(P, s, lane);
-  float2 acc = make_float2(0.f, 0.f);
-  for (int base = cs; base < ce; base += 32) {
-    const int nk = min(32, ce - base);
-    const int jl = lane < nk ? __ldg(rowidx + base + lane) : 0;
-    const float al = lane < nk ? __ldg(val_csc + base + lane) : 0.f;
-    const int ql = lane < nk ? __ldg(perm + base + lane) : 0;
-    for (int k0 = 0; k0 < nk; k0 += kWideBatch) {
-      float2 x[kWideBatch];
-#pragma unroll
-      for (int u = 0; u < kWideBatch; ++u) {
-        const int j = __shfl_sync(FULL_MASK, jl, (k0 + u) & 31);
-        x[u] = (k0 + u < nk) ? ld2(D, j, lane) : make_float2(0.f, 0.f);
-      }
-      float t[kWideBatch];
-#pragma unroll
-      for (int u = 0; u < kWideBatch; ++u) {
-        const float a = __shfl_sync(FULL_MASK, al, (k0 + u) & 31);
-        t[u] = 0.f;
-        if (k0 + u < nk) {   // warp-uniform
-          const int p = base + k0 + u;
-          if (p >= s1) {   // column s is done: report it, move to the column of p
-            vis.segment(s, s0, s1, acc, cs, ce);
-            s = warp_gallop_lower_bound(colptr, s + 1, n + 1, p + 1) - 1;
-            s0 = __ldg(colptr + s);
-            s1 = __ldg(colptr + s + 1);
-            pcol = ld2(P, s, lane);
-            if (kColPrefetchP > 0 && lane < kColPrefetchP && s + 1 + lane < n)
-              prefetch_l2_range(P, (long long)(s + 1 + lane) * 64,
-                                (long long)(s + 2 + lane) * 64);   // the next columns' rows of P
-            acc = make_float2(0.f, 0.f);
-          }
-          acc.x = fmaf(a, x[u].x, acc.x);
-          acc.y = fmaf(a, x[u].y, acc.y);
-          t[u] = fmaf(x[u].y, pcol.y, x[u].x * pcol.x);
-        }
-      }
-      const float r = reduce8(t, lane);   // lane l: key k0 + ((l >> 2) & 7)
-      const int kk = (lane >> 2) & 7;
-      const int q = __shfl_sync(FULL_MASK, ql, (k0 + kk) & 31);
-      if ((lane & 3) == 0 && k0 + kk < nk) dA[q] = r;
-    }
-  }
-  vis.segment(s, s0, s1, acc, cs, ce);
-  *seg_out = s;
-}
-
-// perm != NULL: also dA on the keys (col_walk_sddmm)
-__global__ void __launch_bounds__(kWideThreads)
+// perm != NULL: also dA on the keys
+__global__ void __launch_bounds__(kWideThreads, kWalkCtas)
     gnn_col_kernel(const int32_t* __restrict__ colptr, const int32_t* __restrict__ rowidx,
                    const float* __restrict__ val_csc, int n, int nnz, int nchunks,
                    const float* __restrict__ D, float* __restrict__ G, ChunkPieces pc,
@@ -419,21 +434,28 @@ __global__ void __launch_bounds__(kWideThreads)
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int gw = blockIdx.x * kWideWarps + warp, nw = gridDim.x * kWideWarps;
   const int c0 = (int)(((long long)nchunks * gw) / nw), c1 = (int)(((long long)nchunks * (gw + 1)) / nw);
-  ColVisit vis{G, pc, 0, lane};
+  ColVisit vis;
+  vis.G = G;
+  vis.pc = pc;
+  vis.perm = perm;
+  vis.P = P;
+  vis.dA = dA;
+  vis.n = n;
+  vis.ch = 0;
+  vis.lane = lane;
+  vis.ql = 0;
+  vis.pcol = zero4();
+#pragma unroll
+  for (int u = 0; u < kPairs; ++u) vis.t[u] = 0.f;
   int hint = 0;
   for (int ch = c0; ch < c1; ++ch) {
     const int cs = ch * kWideChunk, ce = min(cs + kWideChunk, nnz);
     if (lane == 0) pc.lastseg[ch] = -1;
     __syncwarp();
     vis.ch = ch;
-    if (cs >= ce) continue;
-    if (perm)
-      col_walk_sddmm(colptr, n, rowidx, val_csc, perm, D, P, dA, cs, ce, hint, lane, vis, &hint);
-    else
-      wide_walk(colptr, n, rowidx, val_csc, D, nnz, cs, ce, hint, lane, vis, &hint);
+    if (cs < ce) pair_walk(colptr, n, rowidx, val_csc, D, cs, ce, hint, lane, vis, &hint);
   }
 }
-
 cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const float* Z,
                     double* loss, float* dA, float* dH, float* dW, const WsLayout& L,
                     cudaStream_t st) {
@@ -464,9 +486,9 @@ cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const flo
   // 2b. forward walk
   {
     KTimer t("gnn_fwd", st);
-    gnn_fwd_kernel<<<g1, kWideThreads, 0, st>>>(A->rowptr, A->colidx, A->val, m, nnz, nchunks,
-                                                 L.P, Z, L.D, dA_in_col ? nullptr : dA, pc,
-                                                 L.hdr, L.partials + ge, loss);
+    auto fwd = (dA && !dA_in_col) ? gnn_fwd_kernel<true> : gnn_fwd_kernel<false>;
+    fwd<<<g1, kWideThreads, 0, st>>>(A->rowptr, A->colidx, A->val, m, nnz, nchunks, L.P, Z, L.D,
+                                     dA_in_col ? nullptr : dA, pc, L.hdr, L.partials + ge, loss);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   // 3. cut rows (also finalises the loss over every partial slot)

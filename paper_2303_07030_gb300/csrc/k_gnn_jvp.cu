@@ -1,0 +1,266 @@
+// k_gnn_jvp.cu -- forward mode of the graph propagation loss (f_out = 64).
+//
+// The loss L = 1/2 |A P - Z|^2 with P = H W, and its derivative along a
+// tangent (A' on A's keys, H', W'), by the forward rules of Sec. 4 with a
+// real tangent: each value carries its tangent through the same steps.
+//   P' = H' W + H W'                               (two tensor-core products)
+//   Y_i  = sum_p A_ip P_j,   Y'_i = sum_p (A'_ip P_j + A_ip P'_j)
+//   D_i  = Y_i - Z_i,        L = 1/2 sum_i |D_i|^2,   L' = sum_i D_i . Y'_i
+// Rows without keys add 1/2 |Z_i|^2 to L and nothing to L'.
+// Kernel sequence: P (and P') on the tensor cores; a walk over the CSR (one
+// warp per 1024-key chunk, one key per step, lane l holding elements 2l,
+// 2l+1 of the rows; P_j and P'_j gathered) whose rows finished inside a
+// chunk add their terms and whose rows cut by chunk boundaries leave pieces
+// of Y and Y'; the rows without keys; a fix kernel that completes the cut
+// rows and adds every CTA's sums in a fixed order.  Reproducible bit for bit.
+#include <algorithm>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace sdad {
+
+constexpr int kGjChunk = kMinCap;
+constexpr int kGjThreads = 256;
+constexpr int kGjWarps = kGjThreads / 32;
+constexpr int kGjBatch = 8;        // keys whose rows are gathered before use
+constexpr int kTangentSlots = kMaxPartials / 2;   // L' partials follow L's
+
+__device__ __forceinline__ float2 gj_ld2(const float* base, int r, int lane) {
+  return __ldg(reinterpret_cast<const float2*>(base + (size_t)r * 64) + lane);
+}
+__device__ __forceinline__ void gj_st2(float* base, int r, int lane, float2 v) {
+  reinterpret_cast<float2*>(base + (size_t)r * 64)[lane] = v;
+}
+__device__ __forceinline__ float gj_wsum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(FULL_MASK, v, o);
+  return v;
+}
+
+struct GjPieces {
+  float* __restrict__ yfirst;   // [chunks x 64]: parts of Y of a row begun earlier
+  float* __restrict__ ylast;    // [chunks x 64]: parts of Y of the row continuing past
+  float* __restrict__ tfirst;   // the same for Y'
+  float* __restrict__ tlast;
+  int* __restrict__ lastseg;
+};
+
+// Stores this CTA's (L, L') sums at slot `slot`.
+__device__ __forceinline__ void gj_publish(double L, double Lt, double* partials, int slot,
+                                           double* red) {
+  const double cL = block_sum_d(L, red);
+  const double cLt = block_sum_d(Lt, red);
+  if (threadIdx.x == 0) {
+    partials[slot] = cL;
+    partials[kTangentSlots + slot] = cLt;
+  }
+}
+
+__global__ void __launch_bounds__(kGjThreads)
+    gnn_jvp_walk_kernel(const int32_t* __restrict__ rowptr, const int32_t* __restrict__ colidx,
+                        const float* __restrict__ val, const float* __restrict__ valt, int m,
+                        int nnz, int nchunks, const float* __restrict__ P,
+                        const float* __restrict__ Pt, const float* __restrict__ Z, GjPieces pc,
+                        double* partials, int first_slot) {
+  __shared__ double red[kGjWarps];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int gw = blockIdx.x * kGjWarps + warp, nw = gridDim.x * kGjWarps;
+  const int c0 = (int)(((long long)nchunks * gw) / nw), c1 = (int)(((long long)nchunks * (gw + 1)) / nw);
+  double L = 0.0, Lt = 0.0;
+  int hint = 0;
+  for (int ch = c0; ch < c1; ++ch) {
+    const int cs = ch * kGjChunk, ce = min(cs + kGjChunk, nnz);
+    if (lane == 0) pc.lastseg[ch] = -1;
+    __syncwarp();
+    if (cs >= ce) continue;
+    int s = warp_gallop_lower_bound(rowptr, hint, m + 1, cs + 1) - 1;
+    int s0 = __ldg(rowptr + s), s1 = __ldg(rowptr + s + 1);
+    float2 y = make_float2(0.f, 0.f), t = y;
+    // the segment s is done: its terms, or its pieces when a chunk boundary cuts it
+    auto close = [&]() {
+      if (s0 >= cs && s1 <= ce) {
+        const float2 z = gj_ld2(Z, s, lane);
+        const float2 d = make_float2(y.x - z.x, y.y - z.y);
+        L += 0.5 * (double)fmaf(d.x, d.x, d.y * d.y);
+        Lt += (double)fmaf(d.x, t.x, d.y * t.y);
+      } else if (s0 < cs) {
+        gj_st2(pc.yfirst, ch, lane, y);
+        gj_st2(pc.tfirst, ch, lane, t);
+      } else {
+        gj_st2(pc.ylast, ch, lane, y);
+        gj_st2(pc.tlast, ch, lane, t);
+        if (lane == 0) pc.lastseg[ch] = s;
+      }
+    };
+    for (int base = cs; base < ce; base += 32) {
+      const int nk = min(32, ce - base);
+      const int jl = lane < nk ? __ldg(colidx + base + lane) : 0;
+      const float al = lane < nk ? __ldg(val + base + lane) : 0.f;
+      const float atl = (valt && lane < nk) ? __ldg(valt + base + lane) : 0.f;
+      for (int k0 = 0; k0 < nk; k0 += kGjBatch) {
+        float2 x[kGjBatch], xt[kGjBatch];
+#pragma unroll
+        for (int u = 0; u < kGjBatch; ++u) {
+          const int j = __shfl_sync(FULL_MASK, jl, (k0 + u) & 31);
+          const bool ok = k0 + u < nk;
+          x[u] = ok ? gj_ld2(P, j, lane) : make_float2(0.f, 0.f);
+          xt[u] = (ok && Pt) ? gj_ld2(Pt, j, lane) : make_float2(0.f, 0.f);
+        }
+#pragma unroll
+        for (int u = 0; u < kGjBatch; ++u) {
+          const float a = __shfl_sync(FULL_MASK, al, (k0 + u) & 31);
+          const float at = __shfl_sync(FULL_MASK, atl, (k0 + u) & 31);
+          if (k0 + u >= nk) break;   // warp-uniform
+          const int p = base + k0 + u;
+          if (p >= s1) {   // row s is done: move to the row of key p
+            close();
+            s = warp_gallop_lower_bound(rowptr, s + 1, m + 1, p + 1) - 1;
+            s0 = __ldg(rowptr + s);
+            s1 = __ldg(rowptr + s + 1);
+            y = make_float2(0.f, 0.f);
+            t = y;
+          }
+          y.x = fmaf(a, x[u].x, y.x);
+          y.y = fmaf(a, x[u].y, y.y);
+          t.x = fmaf(at, x[u].x, fmaf(a, xt[u].x, t.x));
+          t.y = fmaf(at, x[u].y, fmaf(a, xt[u].y, t.y));
+        }
+      }
+    }
+    close();
+    hint = s;
+  }
+  gj_publish(L, Lt, partials, first_slot + blockIdx.x, red);
+}
+
+// rows without keys: L += 1/2 |Z_r|^2 (one warp per 32 rows)
+__global__ void __launch_bounds__(kGjThreads)
+    gnn_jvp_empty_kernel(const int32_t* __restrict__ rowptr, int m, const float* __restrict__ Z,
+                         double* partials) {
+  __shared__ double red[kGjWarps];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int gw = blockIdx.x * kGjWarps + warp, nw = gridDim.x * kGjWarps;
+  double L = 0.0;
+  for (int blk = gw; blk < (m + 31) / 32; blk += nw) {
+    const int r = blk * 32 + lane;
+    const bool e = r < m && __ldg(rowptr + r) == __ldg(rowptr + r + 1);
+    unsigned todo = __ballot_sync(FULL_MASK, e);
+    while (todo) {
+      const int k = __ffs(todo) - 1;
+      todo &= todo - 1;
+      const float2 z = gj_ld2(Z, blk * 32 + k, lane);
+      L += 0.5 * (double)gj_wsum(fmaf(z.x, z.x, z.y * z.y)) * (lane == 0 ? 1.0 : 0.0);
+    }
+  }
+  gj_publish(L, 0.0, partials, blockIdx.x, red);
+}
+
+// rows cut by chunk boundaries, then the totals: the last CTA adds every
+// CTA's sums (slots [0, nslots) of L and of L') in slot order
+__global__ void __launch_bounds__(kGjThreads)
+    gnn_jvp_fix_kernel(const int32_t* __restrict__ rowptr, int nchunks, GjPieces pc,
+                       const float* __restrict__ Z, WsHeader* hdr, double* partials,
+                       int first_slot, double* loss, double* loss_t) {
+  __shared__ double red[kGjWarps];
+  __shared__ bool s_last;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int gw = blockIdx.x * kGjWarps + warp, nw = gridDim.x * kGjWarps;
+  double L = 0.0, Lt = 0.0;
+  for (int ch = gw; ch < nchunks; ch += nw) {
+    const int s = __ldg(pc.lastseg + ch);
+    if (s < 0) continue;   // warp-uniform
+    const int c1 = (__ldg(rowptr + s + 1) - 1) / kGjChunk;
+    float2 y = gj_ld2(pc.ylast, ch, lane), t = gj_ld2(pc.tlast, ch, lane);
+    for (int cc = ch + 1; cc <= c1; ++cc) {
+      const float2 a = gj_ld2(pc.yfirst, cc, lane), b = gj_ld2(pc.tfirst, cc, lane);
+      y.x += a.x;
+      y.y += a.y;
+      t.x += b.x;
+      t.y += b.y;
+    }
+    const float2 z = gj_ld2(Z, s, lane);
+    const float2 d = make_float2(y.x - z.x, y.y - z.y);
+    L += 0.5 * (double)fmaf(d.x, d.x, d.y * d.y);
+    Lt += (double)fmaf(d.x, t.x, d.y * t.y);
+  }
+  gj_publish(L, Lt, partials, first_slot + blockIdx.x, red);
+  if (threadIdx.x == 0) {
+    __threadfence();
+    s_last = atomicAdd(&hdr->ticket, 1u) == gridDim.x - 1;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const int nslots = first_slot + gridDim.x;
+  const volatile double* pv = partials;
+  double a = 0.0, b = 0.0;
+  for (int i = threadIdx.x; i < nslots; i += blockDim.x) {
+    a += pv[i];
+    b += pv[kTangentSlots + i];
+  }
+  a = block_sum_d(a, red);
+  b = block_sum_d(b, red);
+  if (threadIdx.x == 0) {
+    *loss = a;
+    *loss_t = b;
+    hdr->ticket = 0;
+  }
+}
+
+__global__ void add_rows_kernel(float4* __restrict__ a, const float4* __restrict__ b, size_t n4) {
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n4;
+       i += (size_t)gridDim.x * blockDim.x) {
+    const float4 x = a[i], y = __ldg(b + i);
+    a[i] = make_float4(x.x + y.x, x.y + y.y, x.z + y.z, x.w + y.w);
+  }
+}
+
+cudaError_t run_gnn_jvp(const sdad_csr* A, const float* H, const float* W, const float* Z,
+                        const float* valt, const float* Ht, const float* Wt, double* loss,
+                        double* loss_t, const WsLayout& L, cudaStream_t st) {
+  const int sms = device_sm_count();
+  const int m = A->m, n = A->n, nnz = (int)A->nnz;
+  const int nchunks = nnz <= 0 ? 1 : (nnz + kGjChunk - 1) / kGjChunk;
+  cudaError_t e;
+  // P = H W; P' = H' W + H W' (in the G buffer; H W' first goes to D)
+  if ((e = dense_proj_fwd(H, W, L.P, n, L.hdr, st)) != cudaSuccess) return e;
+  const float* Pt = nullptr;
+  if (Ht && (e = dense_proj_fwd(Ht, W, L.G, n, L.hdr, st)) != cudaSuccess) return e;
+  if (Wt) {
+    if ((e = dense_proj_fwd(H, Wt, Ht ? L.D : L.G, n, L.hdr, st)) != cudaSuccess) return e;
+    if (Ht && n > 0) {
+      const size_t n4 = (size_t)n * 16;
+      const int g = (int)std::max<size_t>(1, std::min<size_t>((n4 + 255) / 256, (size_t)sms * 8));
+      KTimer t("gnn_jvp_add", st);
+      add_rows_kernel<<<g, 256, 0, st>>>(reinterpret_cast<float4*>(L.G),
+                                         reinterpret_cast<const float4*>(L.D), n4);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+  }
+  if (Ht || Wt) Pt = L.G;
+  const GjPieces pc{L.pfirst, L.plast, L.tfirst, L.tlast, L.lastseg};
+  const int ge = std::max(1, std::min((m + 255) / 256, sms * 4));
+  {
+    KTimer t("gnn_jvp_empty", st);
+    gnn_jvp_empty_kernel<<<ge, kGjThreads, 0, st>>>(A->rowptr, m, Z, L.partials);
+  }
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  const int gw = std::max(1, std::min((nchunks + kGjWarps - 1) / kGjWarps, sms * 8));
+  {
+    KTimer t("gnn_jvp_walk", st);
+    gnn_jvp_walk_kernel<<<gw, kGjThreads, 0, st>>>(A->rowptr, A->colidx, A->val, valt, m, nnz,
+                                                    nchunks, L.P, Pt, Z, pc, L.partials, ge);
+  }
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  const int gf = std::max(1, std::min((nchunks + kGjWarps - 1) / kGjWarps, sms * 4));
+  static_assert(kTangentSlots >= 152 * 16, "partial slots of the three kernels");
+  {
+    KTimer t("gnn_jvp_fix", st);
+    gnn_jvp_fix_kernel<<<gf, kGjThreads, 0, st>>>(A->rowptr, nchunks, pc, Z, L.hdr, L.partials,
+                                                   ge + gw, loss, loss_t);
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace sdad

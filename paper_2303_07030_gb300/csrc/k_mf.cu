@@ -17,7 +17,10 @@
 // by init_combined.
 #include <algorithm>
 
+#include <climits>
+
 #include "engine.cuh"
+#include "halfwarp.cuh"
 #include "internal.h"
 
 namespace sdad {
@@ -165,9 +168,235 @@ namespace {
 constexpr size_t kMfSmem = pipe_smem_bytes<2, kMfCap, kMfNS>();
 }
 
+// ---------------------------------------------------------------------------
+// One-pass mode (SDAD_T_ATOMIC): a single sweep over the CSR computes e, the
+// loss, dR, dU (row sums in registers) and scatters dV.
+//   init:  dU = 2 lambda U, dV = 2 lambda V (every row), loss part
+//          lambda (|U|^2 + |V|^2)
+//   sweep: one warp per 1024-key chunk, row by row; per batch of 16 keys of
+//          a row, half a warp per key: V_j gathered (16-byte loads), the 16
+//          dot products U_i . V_j reduced together, e = R_ij - U_i . V_j,
+//          dU_i += -2 e V_j in registers, dV_j += -2 e U_i by vector atomic
+//          adds.  With ranked column numbering (sdad_csr_rank_columns) the
+//          kMfHot most used columns are summed in shared memory first and
+//          added to dV once per CTA, so the hottest columns do not serialise
+//          on one address.  Rows cut by chunk boundaries leave pieces.
+//   fix:   dU of the cut rows from their pieces (chunk order); loss total.
+// V rows are gathered once per key instead of twice (row and column pass).
+// The order of the atomic adds varies from run to run.
+constexpr int kMfaChunk = kMinCap;   // the piece slots are per kMinCap keys
+constexpr int kMfaThreads = 256;
+constexpr int kMfaWarps = kMfaThreads / 32;
+constexpr int kMfHot = 64;
+
+__global__ void __launch_bounds__(256)
+    mfa_init_kernel(const float* __restrict__ U, const float* __restrict__ V, int m, int n,
+                    float lam, float* __restrict__ dU, float* __restrict__ dV, WsHeader* hdr,
+                    double* partials) {
+  __shared__ double red[8];
+  const size_t nu = (size_t)m * 16, nt = nu + (size_t)n * 16;   // float4 counts
+  double s = 0.0;
+  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < nt;
+       i += (size_t)gridDim.x * blockDim.x) {
+    const bool u = i < nu;
+    const float4 x = __ldg(reinterpret_cast<const float4*>(u ? U : V) + (u ? i : i - nu));
+    s += (double)dot4(x, x);
+    const float4 g = make_float4(2.f * lam * x.x, 2.f * lam * x.y, 2.f * lam * x.z, 2.f * lam * x.w);
+    if (u) {
+      if (dU) reinterpret_cast<float4*>(dU)[i] = g;
+    } else if (dV) {
+      reinterpret_cast<float4*>(dV)[i - nu] = g;
+    }
+  }
+  const double cta = block_sum_d(s, red);
+  publish_loss(cta * (double)lam, hdr, partials, 0, false, 1.0, nullptr, red);
+}
+
+struct MfaPieces {
+  float* __restrict__ pfirst;   // [chunks x 64]
+  float* __restrict__ plast;    // [chunks x 64]
+  int* __restrict__ lastseg;
+};
+
+__global__ void __launch_bounds__(kMfaThreads)
+    mfa_kernel(const int32_t* __restrict__ rowptr, const int32_t* __restrict__ colidx,
+               const int32_t* __restrict__ rcolidx, const int32_t* __restrict__ rankcol,
+               const float* __restrict__ val, int m, int n, int nnz, int nchunks,
+               const float* __restrict__ U, const float* __restrict__ V, float lam,
+               float* __restrict__ dU, float* __restrict__ dV, float* __restrict__ dR,
+               MfaPieces pc, WsHeader* hdr, double* partials, int first_slot) {
+  __shared__ float hot[kMfHot * 64];
+  __shared__ double red[kMfaWarps];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int h = lane >> 4, sl = lane & 15;
+  const bool ranked = rcolidx != nullptr && dV != nullptr;
+  if (ranked) {
+    for (int i = threadIdx.x; i < kMfHot * 64; i += blockDim.x) hot[i] = 0.f;
+    __syncthreads();
+  }
+  const int gw = blockIdx.x * kMfaWarps + warp, nw = gridDim.x * kMfaWarps;
+  const int c0 = (int)(((long long)nchunks * gw) / nw), c1 = (int)(((long long)nchunks * (gw + 1)) / nw);
+  const int kl = batch_key_of_lane(lane);   // the key whose dot product this lane ends with
+  double loss = 0.0;
+  int hint = 0;
+  for (int ch = c0; ch < c1; ++ch) {
+    const int cs = ch * kMfaChunk, ce = min(cs + kMfaChunk, nnz);
+    if (lane == 0) pc.lastseg[ch] = -1;
+    __syncwarp();
+    if (cs >= ce) continue;
+    int r = warp_gallop_lower_bound(rowptr, hint, m + 1, cs + 1) - 1;   // the row of key cs
+    int s0 = __ldg(rowptr + r), s1 = __ldg(rowptr + r + 1);
+    while (true) {
+      const int ps = max(s0, cs), pe = min(s1, ce);
+      const float4 uv = ld4(U, r, sl);
+      float4 acc = zero4();
+      for (int pb = ps; pb < pe; pb += 2 * kPairs) {
+        const int nk = min(2 * kPairs, pe - pb);
+        const bool mine = lane < nk;
+        const int jl = mine ? __ldg(colidx + pb + lane) : 0;
+        const float al = mine ? __ldg(val + pb + lane) : 0.f;
+        const int rk = (ranked && mine) ? __ldg(rcolidx + pb + lane) : INT_MAX;
+        float4 x[kPairs];
+        float t[kPairs];
+#pragma unroll
+        for (int u = 0; u < kPairs; ++u) {
+          const int kk = 2 * u + h;
+          const int j = __shfl_sync(FULL_MASK, jl, kk);
+          x[u] = kk < nk ? ld4(V, j, sl) : zero4();
+          t[u] = dot4(x[u], uv);
+        }
+        const float d = reduce_half8(t, lane);
+        const float e = __shfl_sync(FULL_MASK, al, kl) - d;   // valid where sl is even and kl < nk
+        if ((sl & 1) == 0 && kl < nk) {
+          loss += (double)e * (double)e;
+          if (dR) dR[pb + kl] = 2.f * e;
+        }
+#pragma unroll
+        for (int u = 0; u < kPairs; ++u) {
+          const int kk = 2 * u + h;
+          const float eu = __shfl_sync(FULL_MASK, e, batch_src_lane(kk));
+          const int j = __shfl_sync(FULL_MASK, jl, kk);
+          const int rank = __shfl_sync(FULL_MASK, rk, kk);
+          if (kk < nk) {
+            acc = fma4(eu, x[u], acc);
+            if (dV) {
+              const float c = -2.f * eu;
+              const float4 g = make_float4(c * uv.x, c * uv.y, c * uv.z, c * uv.w);
+              if (rank < kMfHot) {
+                float* q = hot + rank * 64 + 4 * sl;
+                atomicAdd(q, g.x);
+                atomicAdd(q + 1, g.y);
+                atomicAdd(q + 2, g.z);
+                atomicAdd(q + 3, g.w);
+              } else {
+                atomicAdd(reinterpret_cast<float4*>(dV + (size_t)j * 64) + sl, g);
+              }
+            }
+          }
+        }
+      }
+      const float4 tot = join_halves(acc);
+      if (s0 >= cs && s1 <= ce) {   // the whole row lies in this chunk
+        if (dU && lane < 16) {
+          const float c = 2.f * lam;
+          st4(dU, r, sl, make_float4(fmaf(-2.f, tot.x, c * uv.x), fmaf(-2.f, tot.y, c * uv.y),
+                                     fmaf(-2.f, tot.z, c * uv.z), fmaf(-2.f, tot.w, c * uv.w)));
+        }
+      } else if (lane < 16) {       // a piece of a row cut by the chunk's boundaries
+        if (s0 < cs) {
+          st4(pc.pfirst, ch, sl, tot);
+        } else {
+          st4(pc.plast, ch, sl, tot);
+          if (lane == 0) pc.lastseg[ch] = r;
+        }
+      }
+      if (s1 >= ce) break;
+      // the next row with keys: the one holding key s1
+      r = warp_gallop_lower_bound(rowptr, r + 1, m + 1, s1 + 1) - 1;
+      s0 = __ldg(rowptr + r);
+      s1 = __ldg(rowptr + r + 1);
+    }
+    hint = r;
+  }
+  if (ranked) {   // the hot columns' sums, once per CTA
+    __syncthreads();
+    for (int i = threadIdx.x; i < kMfHot * 64; i += blockDim.x) {
+      const int slot = i >> 6;
+      if (slot < n) atomicAdd(dV + (size_t)__ldg(rankcol + slot) * 64 + (i & 63), hot[i]);
+    }
+  }
+  const double cta = block_sum_d(loss, red);
+  publish_loss(cta, hdr, partials, first_slot, false, 1.0, nullptr, red);
+}
+
+// dU of the rows cut by chunk boundaries: one warp per chunk with a cut row
+// begun in it, its pieces added in chunk order; the last CTA sums the loss.
+__global__ void __launch_bounds__(256)
+    mfa_fix_kernel(const int32_t* __restrict__ rowptr, int nchunks, MfaPieces pc,
+                   const float* __restrict__ U, float lam, float* __restrict__ dU, WsHeader* hdr,
+                   double* partials, int first_slot, double* loss_out) {
+  __shared__ double red[8];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int gw = blockIdx.x * 8 + warp, nw = gridDim.x * 8;
+  for (int ch = gw; ch < nchunks && dU; ch += nw) {
+    const int s = __ldg(pc.lastseg + ch);
+    if (s < 0) continue;   // warp-uniform
+    const int c1 = (__ldg(rowptr + s + 1) - 1) / kMfaChunk;
+    float2 t = __ldg(reinterpret_cast<const float2*>(pc.plast + (size_t)ch * 64) + lane);
+    for (int cc = ch + 1; cc <= c1; ++cc) {
+      const float2 q = __ldg(reinterpret_cast<const float2*>(pc.pfirst + (size_t)cc * 64) + lane);
+      t.x += q.x;
+      t.y += q.y;
+    }
+    const float2 u = __ldg(reinterpret_cast<const float2*>(U + (size_t)s * 64) + lane);
+    reinterpret_cast<float2*>(dU + (size_t)s * 64)[lane] =
+        make_float2(fmaf(-2.f, t.x, 2.f * lam * u.x), fmaf(-2.f, t.y, 2.f * lam * u.y));
+  }
+  publish_loss(0.0, hdr, partials, first_slot, true, 1.0, loss_out, red);
+}
+
+cudaError_t run_mf_atomic(const sdad_csr* R, const float* U, const float* V, float lambda,
+                          double* loss, float* dU, float* dV, float* dR, const WsLayout& L,
+                          cudaStream_t st) {
+  const int sms = device_sm_count();
+  const int m = R->m, n = R->n, nnz = (int)R->nnz;
+  const int nchunks = nnz <= 0 ? 1 : (nnz + kMfaChunk - 1) / kMfaChunk;
+  const size_t n4 = ((size_t)m + (size_t)n) * 16;
+  const int gi = (int)std::max<size_t>(1, std::min<size_t>((n4 + 255) / 256, (size_t)sms * 4));
+  cudaError_t e;
+  {
+    KTimer t("mf_init", st);
+    mfa_init_kernel<<<gi, 256, 0, st>>>(U, V, m, n, lambda, dU, dV, L.hdr, L.partials);
+  }
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  int per_sm = 1;
+  if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, mfa_kernel, kMfaThreads, 0)) !=
+      cudaSuccess)
+    return e;
+  const int gw = std::max(1, std::min((nchunks + kMfaWarps - 1) / kMfaWarps, sms * std::max(per_sm, 1)));
+  const MfaPieces pc{L.pfirst, L.plast, L.lastseg};
+  const bool ranked = csr_ranked(R) && R->rcolidx && R->rankcol;
+  {
+    KTimer t("mf_atomic", st);
+    mfa_kernel<<<gw, kMfaThreads, 0, st>>>(R->rowptr, R->colidx, ranked ? R->rcolidx : nullptr,
+                                            ranked ? R->rankcol : nullptr, R->val, m, n, nnz,
+                                            nchunks, U, V, lambda, dU, dV, dR, pc, L.hdr,
+                                            L.partials, gi);
+  }
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  const int gf = std::max(1, std::min((nchunks + 7) / 8, sms * 8));
+  {
+    KTimer t("mf_fix", st);
+    mfa_fix_kernel<<<gf, 256, 0, st>>>(R->rowptr, nchunks, pc, U, lambda, dU, L.hdr, L.partials,
+                                        gi + gw, loss);
+  }
+  return cudaGetLastError();
+}
+
 cudaError_t run_mf(const sdad_csr* R, const float* U, const float* V, float lambda,
-                   double* loss, float* dU, float* dV, float* dR, sdad_tmode /*tmode*/,
+                   double* loss, float* dU, float* dV, float* dR, sdad_tmode tmode,
                    const WsLayout& L, cudaStream_t st) {
+  if (tmode == SDAD_T_ATOMIC) return run_mf_atomic(R, U, V, lambda, loss, dU, dV, dR, L, st);
   cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void*>(mf_kernel), (int)kMfSmem);
   if (e != cudaSuccess) return e;
   const int sms = device_sm_count();

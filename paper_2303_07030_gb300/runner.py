@@ -120,11 +120,15 @@ class LogregRun(_Base):
 class MfRun(_Base):
     expr = S.SDAD_EXPR_MF
 
-    def __init__(self, p, want_dR=False, device="cuda"):
-        self.p, self.device = p, device
+    def __init__(self, p, want_dR=False, tmode=S.SDAD_T_AUTO, ranked=False, device="cuda"):
+        """tmode: SDAD_T_CSC (row pass + column pass over the CSC twin), SDAD_T_ATOMIC
+        (one pass, dV scattered with atomics; with ranked columns the most used
+        columns are summed in shared memory first) or AUTO (measured)."""
+        self.p, self.device, self.tmode, self.ranked = p, device, tmode, ranked
         self.k = int(p.params["k"])
         self.lam = float(p.params["lam"])
-        self.R = S.CsrDevice(p.m, p.n, p.row, p.col, p.val, csc=True, device=device)
+        self.R = S.CsrDevice(p.m, p.n, p.row, p.col, p.val, csc=True, ranked=ranked,
+                             device=device)
         self.desc = self.R.desc()
         self.U = _dev(p.dense["U"], device)
         self.V = _dev(p.dense["V"], device)
@@ -139,7 +143,11 @@ class MfRun(_Base):
                        self.dR, self.tmode, self.ws, stream)
 
     def step_inputs(self):
-        return _csr_inputs(self.R, self.dV is not None, False) + [self.U, self.V]
+        csc = self.dV is not None and self.tmode != S.SDAD_T_ATOMIC
+        ts = _csr_inputs(self.R, csc, False)
+        if self.ranked:   # the atomic scatter reads the ranks beside the column ids
+            ts += [t for t in (self.R.rcolidx, self.R.rankcol) if t is not None and t.numel()]
+        return ts + [self.U, self.V]
 
     def outputs(self):
         out = {"loss": float(self.loss.item()), "dU": self.dU.cpu().numpy(),

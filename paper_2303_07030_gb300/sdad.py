@@ -38,7 +38,7 @@ EXPORTS = [
     "sdad_smvm_grad", "sdad_smmm_grad", "sdad_csr_gram_pattern",
     "sdad_batax_grad",
     "sdad_timing_enable", "sdad_timing_reset", "sdad_timing_count", "sdad_timing_get",
-    "sdad_probe_fma",
+    "sdad_probe_fma", "sdad_gather_by_perm", "sdad_gnn_jvp",
 ]
 
 
@@ -121,6 +121,9 @@ def lib():
             "sdad_timing_count": ([], i32),
             "sdad_timing_get": ([i32, P(ctypes.c_char_p), P(ctypes.c_float)], i32),
             "sdad_probe_fma": ([vp, i32, i32, P(ctypes.c_double), vp], i32),
+            "sdad_gather_by_perm": ([vp, i64, vp, i64, vp, vp], i32),
+            "sdad_gnn_jvp": ([P(sdad_csr), vp, vp, vp, i32, i32, vp, vp, vp, vp, vp, vp, sz, vp],
+                             i32),
         }
         for name, (args, res) in sigs.items():
             fn = getattr(L, name)
@@ -321,6 +324,14 @@ def sdad_timing_records():
     return [sdad_timing_get(i) for i in range(sdad_timing_count())]
 
 
+def sdad_gather_by_perm(src, perm, out, stream=None):
+    """out[q] = src[perm[q]] (0 where perm[q] is out of range), on the device; 4-byte dtypes."""
+    assert src.element_size() == 4 and out.element_size() == 4 and perm.numel() == out.numel()
+    _check(lib().sdad_gather_by_perm(_ptr(src), src.numel(), _ptr(perm), perm.numel(), _ptr(out),
+                                     _stream(stream)), "sdad_gather_by_perm")
+    return out
+
+
 def sdad_probe_fma(out, blocks, iters, stream=None):
     """Enqueues the FP32 FMA probe; returns the FLOPs it performs."""
     fl = ctypes.c_double(0.0)
@@ -359,16 +370,18 @@ class CsrDevice:
             else:
                 colptr, rowidx, perm = sdad_csr_transpose(m, n, rowptr, colidx)
             self.colptr, self.rowidx, self.perm = dev(colptr), dev(rowidx), dev(perm)
-            self.val_csc = self.val[self.perm.long()].contiguous()
+            self.val_csc = torch.empty(perm.size, dtype=torch.float32, device=device)
+            sdad_gather_by_perm(self.val, self.perm, self.val_csc)
             self.host.update(colptr=colptr, rowidx=rowidx, perm=perm)
         self.bcsc_log2, self.bcsc_nnz, self.bcsc_ncols = 0, 0, 0
-        self.bcsc_ptr = self.bcsc_key = self.bcsc_val = self.bcsc_cols = None
+        self.bcsc_ptr = self.bcsc_key = self.bcsc_val = self.bcsc_cols = self.bperm = None
         if blocked:
             # row-blocked CSC twin with 2^blocked rows per block
             bp, bk, bperm = sdad_csr_block_transpose(m, n, rowptr, colidx, blocked, block_cols)
-            bval = np.where(bperm >= 0, v[np.maximum(bperm, 0)], 0).astype(np.float32)
             self.bcsc_log2, self.bcsc_nnz = int(blocked), int(bk.size)
-            self.bcsc_ptr, self.bcsc_key, self.bcsc_val = dev(bp), dev(bk.view(np.int32)), dev(bval)
+            self.bcsc_ptr, self.bcsc_key, self.bperm = dev(bp), dev(bk.view(np.int32)), dev(bperm)
+            self.bcsc_val = torch.empty(bk.size, dtype=torch.float32, device=device)
+            sdad_gather_by_perm(self.val, self.bperm, self.bcsc_val)
             self.host.update(bcsc_ptr=bp, bcsc_key=bk, bcsc_perm=bperm)
             if split:
                 bc = np.ascontiguousarray(block_cols, dtype=np.int32)
@@ -380,6 +393,14 @@ class CsrDevice:
             rcol, rankcol = sdad_csr_rank_columns(n, colidx)
             self.rcolidx, self.rankcol = dev(rcol), dev(rankcol)
             self.host.update(rcolidx=rcol, rankcol=rankcol)
+
+    def refresh_values(self, stream=None):
+        """After self.val changed on the device: the twins' value copies again
+        (val_csc = val[perm], bcsc_val = val[bperm]), gathered on the device."""
+        if self.val_csc is not None and self.perm is not None:
+            sdad_gather_by_perm(self.val, self.perm, self.val_csc, stream)
+        if self.bcsc_val is not None and self.bperm is not None:
+            sdad_gather_by_perm(self.val, self.bperm, self.bcsc_val, stream)
 
     def desc(self):
         return sdad_csr(self.m, self.n, self.nnz, _ptr(self.rowptr), _ptr(self.colidx),
@@ -410,9 +431,11 @@ class Coo3Device:
             perm, seg = sdad_coo3_mode_index(host_idx[0], host_idx[1], host_idx[2], self.dims, m)
             self.sperm[m] = dev(perm)
             self.segptr[m] = dev(seg)
+            # the sorted copies, gathered on the device through the mode's permutation
             for c in range(3):
-                self.sidx[m][c] = dev(host_idx[c][perm])
-            self.sval[m] = dev(host_val[perm])
+                self.sidx[m][c] = sdad_gather_by_perm(self.idx[c], self.sperm[m],
+                                                      torch.empty_like(self.idx[c]))
+            self.sval[m] = sdad_gather_by_perm(self.val, self.sperm[m], torch.empty_like(self.val))
 
     def desc(self):
         d = sdad_coo3()
@@ -502,6 +525,15 @@ def sdad_mf_jvp(R, U, V, k, lam, loss, loss_t, R_t_val=None, U_t=None, V_t=None,
     _check(lib().sdad_mf_jvp(ctypes.byref(d), _ptr(U), _ptr(V), k, float(lam), _ptr(R_t_val),
                              _ptr(U_t), _ptr(V_t), _ptr(loss), _ptr(loss_t), wp, wb,
                              _stream(stream)), "sdad_mf_jvp")
+
+
+def sdad_gnn_jvp(A, H, W, Z, f_in, f_out, loss, loss_t, A_t_val=None, H_t=None, W_t=None,
+                 ws=None, stream=None):
+    d = A.desc() if hasattr(A, "desc") else A
+    wp, wb = _ws(ws)
+    _check(lib().sdad_gnn_jvp(ctypes.byref(d), _ptr(H), _ptr(W), _ptr(Z), f_in, f_out,
+                              _ptr(A_t_val), _ptr(H_t), _ptr(W_t), _ptr(loss), _ptr(loss_t), wp,
+                              wb, _stream(stream)), "sdad_gnn_jvp")
 
 
 def sdad_cp3_jvp(T, A, B, C, rank, loss, loss_t, T_t_val=None, A_t=None, B_t=None, C_t=None,

@@ -72,8 +72,8 @@ def test_flops_and_traffic_tables():
     p = W.make("mf", "small")
     f = bench.kernel_flops("mf", p, p.nnz)
     assert f["mf_row"] == 256 * p.nnz and f["mf_atomic"] == 384 * p.nnz
-    g = W.make("gnn", "small")
-    assert bench.kernel_flops("gnn", g, g.nnz)["proj_dw"] == 2 * g.n * 128 * 64
+    c = W.make("cp3", "small")
+    assert bench.kernel_flops("cp3", c, c.nnz)["cp_atomic"] == 384 * c.nnz
     # a figure is given only for the layout it was captured on
     lay = dict(bench.NCU_TRAFFIC["logreg"]["layout"])
     t, src = bench.measured_traffic("logreg", "logreg_row", 1000, lay)

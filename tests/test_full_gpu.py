@@ -35,15 +35,16 @@ def _problem_and_oracle(name):
 # row-blocked CSC twin of every column with 2^15-row blocks: 31 blocks), the
 # ranked columns with the plain CSC twin, the split column pass (blocked
 # columns with >= 32 keys per 2^15-row block), the atomic transposed product,
-# and the columns as generated; CP with its one-pass atomic scatter (AUTO) and
-# with the sorted per-mode passes (SDAD_T_CSC)
+# and the columns as generated; MF with its two passes (SDAD_T_CSC) and with
+# the one-pass atomic scatter over ranked columns; CP with its one-pass atomic
+# scatter (AUTO) and with the sorted per-mode passes (SDAD_T_CSC)
 @pytest.mark.parametrize("name,kw", [
     ("logreg", {"ranked": True, "blocked": 15}),
     ("logreg", {"ranked": True}),
     ("logreg", {"ranked": True, "split": (15, 32.0)}),
     ("logreg", {"ranked": True, "tmode": 2}),
     ("logreg", {}),
-    ("mf", {}),
+    ("mf", {"tmode": 1}), ("mf", {"tmode": 2, "ranked": True}),
     ("cp3", {}), ("cp3", {"tmode": 1}),
     ("gnn", {}),
 ])

@@ -249,3 +249,82 @@ def test_mf_cp3_jvp_full_size():
     g = oracle.cp3(p.dims, p.i, p.j, p.k, p.val, p.dense["A"], p.dense["B"], p.dense["C"])
     assert abs(L - ref["loss"]) <= TOL * abs(ref["loss"])
     assert abs(Lt - ref["loss_t"]) <= TOL * _sbound([(g["dT"], tt)])
+
+
+# ----------------------------------------------------------------------------
+# graph propagation: P' = H' W + H W' on the tensor cores, Y' = A' P + A P'
+# ----------------------------------------------------------------------------
+
+def _jvp_gnn(run, valt, Ht, Wt):
+    out = torch.zeros(2, dtype=torch.float64, device="cuda")
+    S.sdad_gnn_jvp(run.desc, run.H, run.W, run.Z, run.f_in, run.f_out, out[0:], out[1:],
+                   dev(valt), dev(Ht), dev(Wt), run.ws)
+    torch.cuda.synchronize()
+    run.check()
+    o = out.cpu().numpy()
+    return float(o[0]), float(o[1])
+
+
+def _gnn_tangents(rng, p):
+    return (rng.standard_normal(p.nnz).astype(np.float32),
+            rng.standard_normal(p.dense["H"].shape).astype(np.float32),
+            (0.1 * rng.standard_normal(p.dense["W"].shape)).astype(np.float32))
+
+
+@pytest.mark.parametrize("parts", ["all", "values", "H", "W"])
+def test_gnn_jvp_against_oracle_and_reverse_mode(parts):
+    p = W.make("gnn", "small")
+    rng = np.random.default_rng(15)
+    valt, Ht, Wt = _gnn_tangents(rng, p)
+    valt = valt if parts in ("all", "values") else None
+    Ht = Ht if parts in ("all", "H") else None
+    Wt = Wt if parts in ("all", "W") else None
+    run = R.GnnRun(p)
+    L, Lt = _jvp_gnn(run, valt, Ht, Wt)
+    d = p.dense
+    ref = oracle.gnn_jvp(p.m, p.n, p.row, p.col, p.val, d["H"], d["W"], d["Z"], valt, Ht, Wt)
+    g = oracle.gnn(p.m, p.n, p.row, p.col, p.val, d["H"], d["W"], d["Z"])
+    b = _sbound([(g["dA"], valt), (g["dH"], Ht), (g["dW"], Wt)])
+    assert abs(L - ref["loss"]) <= TOL * abs(ref["loss"])
+    assert abs(Lt - ref["loss_t"]) <= TOL * b
+    # adjoint identity with the GPU's reverse mode
+    run.step()
+    torch.cuda.synchronize()
+    run.check()
+    o = run.outputs()
+    dot = sum(float((o[k].astype(np.float64) * t).sum())
+              for k, t in (("dA", valt), ("dH", Ht), ("dW", Wt)) if t is not None)
+    assert abs(Lt - dot) <= TOL * b
+    assert _jvp_gnn(run, valt, Ht, Wt) == (L, Lt)   # reproducible
+
+
+def test_gnn_jvp_zero_tangent_and_empty_rows():
+    p = W.make("gnn", "small")
+    run = R.GnnRun(p)
+    L0, Lt0 = _jvp_gnn(run, None, None, None)
+    d = p.dense
+    ref = oracle.gnn_jvp(p.m, p.n, p.row, p.col, p.val, d["H"], d["W"], d["Z"])
+    assert Lt0 == 0.0 and abs(L0 - ref["loss"]) <= TOL * abs(ref["loss"])
+    # a matrix without keys: L = 1/2 |Z|^2, L' = 0 whatever the tangent
+    e = np.zeros(0, np.int32)
+    q = W.SparseMatrixProblem("gnn", p.m, p.n, e, e, np.zeros(0, np.float32), p.dense, p.params)
+    run0 = R.GnnRun(q)
+    rng = np.random.default_rng(16)
+    _, Ht, Wt = _gnn_tangents(rng, p)
+    L, Lt = _jvp_gnn(run0, None, Ht, Wt)
+    z = d["Z"].astype(np.float64)
+    assert abs(L - 0.5 * (z * z).sum()) <= 1e-6 * L and Lt == 0.0
+
+
+@pytest.mark.full
+def test_gnn_jvp_full_size():
+    p = W.make("gnn", "full")
+    rng = np.random.default_rng(17)
+    valt, _, Wt = _gnn_tangents(rng, p)
+    run = R.GnnRun(p)
+    L, Lt = _jvp_gnn(run, valt, None, Wt)
+    d = p.dense
+    ref = oracle.gnn_jvp(p.m, p.n, p.row, p.col, p.val, d["H"], d["W"], d["Z"], valt, None, Wt)
+    g = oracle.gnn(p.m, p.n, p.row, p.col, p.val, d["H"], d["W"], d["Z"])
+    assert abs(L - ref["loss"]) <= TOL * abs(ref["loss"])
+    assert abs(Lt - ref["loss_t"]) <= TOL * _sbound([(g["dA"], valt), (g["dW"], Wt)])

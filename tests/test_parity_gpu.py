@@ -83,11 +83,33 @@ def test_logreg_small(tmode):
     assert_close(out, ref, ["dw", "dX"])
 
 
-def test_mf_small():
+# the two-pass path over the CSC twin, the one-pass atomic scatter (with and
+# without the ranked numbering that sums the hot columns in shared memory),
+# and AUTO (both timed on the first call, the faster kept)
+@pytest.mark.parametrize("kw", [{"tmode": S.SDAD_T_CSC}, {"tmode": S.SDAD_T_ATOMIC},
+                                {"tmode": S.SDAD_T_ATOMIC, "ranked": True},
+                                {"tmode": S.SDAD_T_AUTO, "ranked": True}])
+def test_mf_small(kw):
     p = W.make("mf", "small")
-    r, out = run("mf", p, want_dR=True)
+    r, out = run("mf", p, want_dR=True, **kw)
     pattern_matches(r, p)
     assert_close(out, oracle_for("mf", p), ["dU", "dV", "dR"])
+    if kw["tmode"] == S.SDAD_T_AUTO:   # the kept choice on a second call
+        r.step()
+        torch.cuda.synchronize()
+        r.check()
+        assert_close(r.outputs(), oracle_for("mf", p), ["dU", "dV", "dR"])
+
+
+def test_mf_atomic_without_csc_twin():
+    # AUTO on a matrix without its CSC twin takes the one-pass scatter
+    p = W.make("mf", "small")
+    r = R.MfRun(p)
+    r.desc.colptr = r.desc.rowidx = r.desc.val_csc = None
+    r.step()
+    torch.cuda.synchronize()
+    r.check()
+    assert_close(r.outputs(), oracle_for("mf", p), ["dU", "dV"])
 
 
 @pytest.mark.parametrize("tmode", [S.SDAD_T_CSC, S.SDAD_T_ATOMIC])
@@ -160,7 +182,9 @@ def test_logreg_hot_column_across_chunks():
         assert_close(out, oracle_for("logreg", p), ["dw", "dX"])
 
 
-def test_mf_hub_row_and_column():
+@pytest.mark.parametrize("kw", [{"tmode": S.SDAD_T_CSC},
+                                {"tmode": S.SDAD_T_ATOMIC, "ranked": True}])
+def test_mf_hub_row_and_column(kw):
     rng = np.random.default_rng(4)
     m, n, k = 400, 6000, 64
     row = np.concatenate([np.zeros(5500, np.int64), rng.integers(0, m, 9000),
@@ -173,7 +197,7 @@ def test_mf_hub_row_and_column():
                {"U": (0.1 * rng.standard_normal((m, k))).astype(np.float32),
                 "V": (0.1 * rng.standard_normal((n, k))).astype(np.float32)},
                {"k": k, "lam": 0.01})
-    _, out = run("mf", p, want_dR=True)
+    _, out = run("mf", p, want_dR=True, **kw)
     assert_close(out, oracle_for("mf", p), ["dU", "dV", "dR"])
 
 
