@@ -85,6 +85,11 @@ def parse():
                     help="lsq/logreg: column numbering of the matrix (ranked by key count, "
                          "built once on the host, or as generated; auto: ranked for the "
                          "Zipf-skewed logistic columns, as generated for the uniform lsq ones)")
+    ap.add_argument("--sweep", action="store_true",
+                    help="instead of the benchmark line: the density / dimension sweep of the "
+                         "library's own passes (least squares at fixed dimension and at fixed "
+                         "keys per row, logistic regression by keys per row, R-MAT graphs by "
+                         "scale); one JSON line with a point per instance")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--override", action="append", default=[], metavar="KEY=VALUE",
@@ -619,8 +624,84 @@ def measure(cfg, args, ov, dist, world, local, headline, fma):
     return p, res
 
 
+SWEEP = [
+    # (workload, generator overrides, what varies)
+    ("lsq", dict(m=1 << 20, n=1 << 20, draws=1 << 20), "density"),
+    ("lsq", dict(m=1 << 20, n=1 << 20, draws=1 << 22), "density"),
+    ("lsq", dict(m=1 << 20, n=1 << 20, draws=1 << 24), "density"),
+    ("lsq", dict(m=1 << 20, n=1 << 20, draws=1 << 26), "density"),
+    ("lsq", dict(m=1 << 16, n=1 << 16, draws=1 << 20), "dimension"),
+    ("lsq", dict(m=1 << 18, n=1 << 18, draws=1 << 22), "dimension"),
+    ("lsq", dict(m=1 << 22, n=1 << 22, draws=1 << 26), "dimension"),
+    ("logreg", dict(mean_row=10.0), "density"),
+    ("logreg", dict(mean_row=25.0), "density"),
+    ("logreg", dict(mean_row=100.0), "density"),
+    ("gnn", dict(scale=16, n_edges=1 << 20), "dimension"),
+    ("gnn", dict(scale=18, n_edges=1 << 22), "dimension"),
+    ("gnn", dict(scale=20, n_edges=1 << 24), "dimension"),
+]
+
+
+def run_sweep(args):
+    """Density and dimension sweep of the library's own passes (no comparison system)."""
+    import torch
+    from paper_2303_07030_gb300 import build as B
+    from paper_2303_07030_gb300 import sdad as S
+    from paper_2303_07030_gb300 import workloads as W
+    B.build()
+    hbm, src = peaks()
+    stream = torch.cuda.current_stream()
+    points = []
+    for cfg, ov, what in SWEEP:
+        p = W.make(cfg, "full", **ov)
+        ranked, blocked, block_cols, split, transpose = layout_for(cfg, p, args, S)
+        run = make_run(cfg, p, "auto", ranked, blocked, block_cols)
+        for _ in range(3):
+            run.step()
+        torch.cuda.synchronize()
+        run.check()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(10):
+            run.step()
+        b.record(stream)
+        torch.cuda.synchronize()
+        ms = a.elapsed_time(b) / 10
+        S.sdad_timing_reset()
+        S.sdad_timing_enable(True)
+        for _ in range(5):
+            run.step()
+        torch.cuda.synchronize()
+        S.sdad_timing_enable(False)
+        run.check()
+        per = {}
+        for name, kms in S.sdad_timing_records():
+            per.setdefault(name, []).append(kms)
+        csc = getattr(run, "csc", True)
+        kb = kernel_bytes(cfg, p, p.nnz, csc, False, ranked, blocked, split)
+        tot = sum(kb.get(k, 0) * len(v) for k, v in per.items()) / 5
+        dom = max((k for k in per if k in kb), key=lambda k: sum(per[k]), default=None)
+        pt = {"workload": cfg, "varies": what, "params": ov, "m": p.m, "n": p.n, "nnz": p.nnz,
+              "density": p.nnz / (float(p.m) * p.n), "ms_per_step": round(ms, 5),
+              "value": p.nnz / (ms * 1e-3), "hbm_gbs_step": round(tot / (ms * 1e-3) / 1e9, 1)}
+        if dom is not None:
+            dms = sum(per[dom]) / len(per[dom])
+            pt["dominant"] = {"kernel": dom, "ms": round(dms, 5),
+                              "frac": round(kb[dom] / (dms * 1e-3) / 1e9 / hbm, 4)}
+        points.append(pt)
+        print(json.dumps(pt), file=sys.stderr, flush=True)
+        del run
+        torch.cuda.empty_cache()
+    print(json.dumps({"metric": METRIC, "unit": UNIT, "sweep": points, "peak_gbs": hbm,
+                      "peak_source": src, "data": "synthetic (seeded generators)"}), flush=True)
+    return 0
+
+
 def main():
     args = parse()
+    if args.sweep and args.impl == "ours":
+        return run_sweep(args)
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local = int(os.environ.get("LOCAL_RANK", "0"))

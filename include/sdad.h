@@ -245,6 +245,17 @@ typedef struct {
   const int32_t* csc_perm;  /* device int32[nnz], or NULL */
 } sdad_csr;
 
+/* Sparse matrix A (m x n) as COO entries in any order (Sec. 5.3, Fig.
+ * "storage_spec": the coordinate format of the same dictionary).  Entries may
+ * repeat a key; their values add. */
+typedef struct {
+  int32_t m, n;
+  int64_t nnz;
+  const int32_t* row;   /* device int32[nnz], each in [0, m) */
+  const int32_t* col;   /* device int32[nnz], each in [0, n) */
+  const float* val;     /* device float[nnz]                 */
+} sdad_coo;
+
 /* 3-way sparse tensor in COO plus one mode-sorted copy per mode. */
 typedef struct {
   int32_t dims[3];
@@ -335,6 +346,19 @@ sdad_status sdad_workspace_set_wait_limit(void* ws, int64_t polls, void* stream)
 sdad_status sdad_lsq_grad(const sdad_csr* A, const float* x, const float* y, double* loss,
                           float* dx, float* dA_val, sdad_tmode tmode, void* ws, size_t ws_bytes,
                           void* stream);
+
+/* Least squares as sdad_lsq_grad over a COO operand in entry order (no CSR,
+ * no twins, no sorting): z = A x by an entry scatter, r = z - y and the loss
+ * by a row pass, then dA and dx = A^T r by a second entry pass.  dA_val[nnz]
+ * is in the entries' order (an entry that repeats a key gets the key's
+ * gradient r_i x_j).  The scatters use warp-aggregated float atomics, so dx
+ * (and z) are order-dependent within rounding; the loss is summed in a fixed
+ * order.  Indices are checked on the device: an entry out of range is skipped
+ * and SDAD_ERR_INDEX is recorded for sdad_check.  Workspace: as
+ * sdad_lsq_grad (sdad_workspace_bytes(SDAD_EXPR_LSQ, m, n, nnz, 0)).
+ * Errors: NULL/SHAPE/ALIGN/OVERFLOW/WORKSPACE/CUDA. */
+sdad_status sdad_lsq_coo_grad(const sdad_coo* A, const float* x, const float* y, double* loss,
+                              float* dx, float* dA_val, void* ws, size_t ws_bytes, void* stream);
 
 /* Logistic regression over m samples (rows of X: m x n), labels y in [0, 1]:
  *   z = X w,  L = (1/m) sum_i [log(1 + e^{z_i}) - y_i z_i]

@@ -427,6 +427,21 @@ sdad_status sdad_lsq_grad(const sdad_csr* A, const float* x, const float* y, dou
   return scalar_entry(SDAD_EXPR_LSQ, A, x, y, loss, dx, dA_val, tmode, ws, ws_bytes, stream);
 }
 
+sdad_status sdad_lsq_coo_grad(const sdad_coo* A, const float* x, const float* y, double* loss,
+                              float* dx, float* dA_val, void* ws, size_t ws_bytes, void* stream) {
+  if (!A || !loss) return SDAD_ERR_NULL;
+  if (A->m < 0 || A->n < 0 || A->nnz < 0) return SDAD_ERR_SHAPE;
+  if (A->nnz > kMaxNnz) return SDAD_ERR_OVERFLOW;
+  if (A->nnz > 0 && (!A->row || !A->col || !A->val)) return SDAD_ERR_NULL;
+  if ((!x && A->n > 0) || (!y && A->m > 0)) return SDAD_ERR_NULL;
+  if (!a8(loss)) return SDAD_ERR_ALIGN;
+  const WsLayout L = ws_layout(SDAD_EXPR_LSQ, A->m, A->n, A->nnz, 0, ws);
+  sdad_status s;
+  if ((s = check_ws(L, ws, ws_bytes))) return s;
+  if ((s = check_device())) return s;
+  return map_cuda(run_lsq_coo(A, x, y, loss, dx, dA_val, L, (cudaStream_t)stream));
+}
+
 sdad_status sdad_logreg_grad(const sdad_csr* X, const float* w, const float* y, double* loss,
                              float* dw, float* dX_val, sdad_tmode tmode, void* ws,
                              size_t ws_bytes, void* stream) {

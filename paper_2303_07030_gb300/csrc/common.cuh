@@ -181,6 +181,26 @@ __device__ __forceinline__ double warp_sum_d(double v) {
   return v;
 }
 
+// base[idx] += v with one atomic per distinct idx among the calling lanes
+// (idx < 0: nothing is added for that lane):
+// `active` must be exactly the lanes that call it.  Lanes with equal idx
+// (found with __match_any_sync) add their values in lane order and the
+// lowest of them issues the atomic, so a hot index costs one atomic per warp
+// instead of one per lane.  The shuffles run over `peers`, the lanes that
+// share an index, all of which execute the same loop.
+__device__ __forceinline__ void agg_atomic_add(float* base, int idx, float v, unsigned active) {
+  const unsigned peers = __match_any_sync(active, idx);
+  const int lane = threadIdx.x & 31;
+  if (idx < 0) return;
+  if (peers == (1u << lane)) {
+    atomicAdd(base + idx, v);
+    return;
+  }
+  float s = 0.f;
+  for (unsigned m = peers; m; m &= m - 1) s += __shfl_sync(peers, v, __ffs(m) - 1);
+  if (lane == __ffs(peers) - 1) atomicAdd(base + idx, s);
+}
+
 // First i in [lo, hi) with ptr[i] >= key, or hi if none.  ptr is
 // non-decreasing.  Called by a full warp; every lane gets the answer.
 __device__ __forceinline__ int warp_lower_bound(const int32_t* __restrict__ ptr, int lo, int hi,

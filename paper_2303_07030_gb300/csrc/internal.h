@@ -112,6 +112,9 @@ cudaError_t run_cp3(const sdad_coo3* T, const float* A, const float* B, const fl
                     double* loss, float* dA, float* dB, float* dC, float* dT, sdad_tmode tmode,
                     const WsLayout& L, cudaStream_t st);
 
+cudaError_t run_lsq_coo(const sdad_coo* A, const float* x, const float* y, double* loss,
+                        float* dx, float* dA, const WsLayout& L, cudaStream_t st);
+
 cudaError_t run_gnn_jvp(const sdad_csr* A, const float* H, const float* W, const float* Z,
                         const float* valt, const float* Ht, const float* Wt, double* loss,
                         double* loss_t, const WsLayout& L, cudaStream_t st);

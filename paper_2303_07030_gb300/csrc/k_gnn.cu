@@ -37,6 +37,10 @@ namespace sdad {
 constexpr int kWideChunk = kMinCap;   // 1024 keys: the piece slots are per kMinCap keys
 constexpr int kWideThreads = 256;
 constexpr int kWideWarps = kWideThreads / 32;
+#ifndef SDAD_WALK_LOOKAHEAD
+#define SDAD_WALK_LOOKAHEAD 1
+#endif
+constexpr bool kWalkLookahead = SDAD_WALK_LOOKAHEAD;   // next row's Z / next column's P loaded ahead
 constexpr int kWalkCtas = 3;          // resident CTAs per SM the walks are compiled for (<= 85 registers)
 
 __device__ __forceinline__ float2 ld2(const float* base, int r, int lane) {
@@ -52,6 +56,7 @@ __device__ __forceinline__ void st2(float* base, int r, int lane, float2 v) {
 // beyond them, a binary search.  Called by the whole warp.
 struct Seg {
   int s, s0, s1;
+  int after;   // the segment after s that holds keys, when it lies in the same 32 pointers; else -1
 };
 __device__ __forceinline__ Seg next_segment(const int32_t* __restrict__ ptr, int nseg, int lo,
                                             int p, int lane) {
@@ -63,11 +68,14 @@ __device__ __forceinline__ Seg next_segment(const int32_t* __restrict__ ptr, int
     const int f = __ffs(b) - 1;
     const int s1 = __shfl_sync(FULL_MASK, pv, f);
     const int before = __shfl_sync(FULL_MASK, pv, (f + 31) & 31);
+    // the segment holding key s1: the last i with ptr[i] <= s1
+    const unsigned b2 = __ballot_sync(FULL_MASK, pv > s1 && pv != INT_MAX);
+    const int after = (kWalkLookahead && b2) ? lo + __ffs(b2) - 1 : -1;
     // f = 0 would mean p lies in segment lo itself (not so where the walks call this)
-    return Seg{lo + f, f ? before : __ldg(ptr + lo), s1};
+    return Seg{lo + f, f ? before : __ldg(ptr + lo), s1, after};
   }
   const int s = warp_lower_bound(ptr, lo + 33, nseg + 1, p + 1) - 1;
-  return Seg{s, __ldg(ptr + s), __ldg(ptr + s + 1)};
+  return Seg{s, __ldg(ptr + s), __ldg(ptr + s + 1), -1};
 }
 
 struct ChunkPieces {
@@ -108,7 +116,7 @@ __device__ __forceinline__ void pair_walk(const int32_t* __restrict__ ptr, int n
   // the segment holding key cs: the last s with ptr[s] <= cs
   int s = warp_gallop_lower_bound(ptr, hint, nseg + 1, cs + 1) - 1;
   int s0 = __ldg(ptr + s), s1 = __ldg(ptr + s + 1);
-  vis.begin(s, lane);
+  vis.begin(s, -1);
   float4 acc = zero4();
   for (int base = cs; base < ce; base += 32) {
     const int nk = min(32, ce - base);
@@ -140,7 +148,7 @@ __device__ __forceinline__ void pair_walk(const int32_t* __restrict__ ptr, int n
           vis.segment(s, s0, s1, join_halves(acc), cs, ce);
           const Seg g = next_segment(ptr, nseg, s, p0, lane);
           s = g.s; s0 = g.s0; s1 = g.s1;
-          vis.begin(s, lane);
+          vis.begin(s, g.after);
           acc = zero4();
         }
         if (h == 0) acc = fma4(a, x[u], acc);
@@ -150,7 +158,7 @@ __device__ __forceinline__ void pair_walk(const int32_t* __restrict__ ptr, int n
             vis.segment(s, s0, s1, join_halves(acc), cs, ce);
             const Seg g = next_segment(ptr, nseg, s, p0 + 1, lane);
             s = g.s; s0 = g.s0; s1 = g.s1;
-            vis.begin(s, lane);
+            vis.begin(s, g.after);
             acc = zero4();
           }
           if (h == 1) acc = fma4(a, x[u], acc);
@@ -204,8 +212,16 @@ struct FwdVisit {
   ChunkPieces pc;
   int ch, lane;
   double loss;   // this lane's part
+  float4 zr;     // Z row of the open row (loaded when the row begins)
+  float4 znext;  // Z row of row znext_r, loaded one row ahead
+  int znext_r;
 
-  __device__ __forceinline__ void begin(int, int) {}
+  __device__ __forceinline__ void begin(int r, int after) {
+    const int sl = lane & 15;
+    zr = r == znext_r ? znext : ld4(Z, r, sl);
+    znext_r = after;
+    if (after >= 0) znext = ld4(Z, after, sl);
+  }
   __device__ __forceinline__ void window(int, int, int) {}
   __device__ __forceinline__ void key(int, float4, int, int) {}
   __device__ __forceinline__ void key_if(bool, float4, int, int) {}
@@ -213,8 +229,7 @@ struct FwdVisit {
   __device__ __forceinline__ void segment(int r, int s0, int s1, float4 tot, int cs, int ce) {
     if (pc.cut(ch, r, s0, s1, cs, ce, tot, lane)) return;
     const int sl = lane & 15;
-    const float4 z = ld4(Z, r, sl);
-    const float4 d = make_float4(tot.x - z.x, tot.y - z.y, tot.z - z.z, tot.w - z.w);
+    const float4 d = make_float4(tot.x - zr.x, tot.y - zr.y, tot.z - zr.z, tot.w - zr.w);
     if (lane < 16) {
       st4(D, r, sl, d);
       loss += 0.5 * (double)dot4(d, d);
@@ -237,7 +252,7 @@ __global__ void __launch_bounds__(kWideThreads, kWalkCtas)
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int gw = blockIdx.x * kWideWarps + warp, nw = gridDim.x * kWideWarps;
   const int c0 = (int)(((long long)nchunks * gw) / nw), c1 = (int)(((long long)nchunks * (gw + 1)) / nw);
-  FwdVisit vis{colidx, P, Z, D, WITH_DA ? dA : nullptr, pc, 0, lane, 0.0};
+  FwdVisit vis{colidx, P, Z, D, WITH_DA ? dA : nullptr, pc, 0, lane, 0.0, zero4(), zero4(), -1};
   int hint = 0;
   for (int ch = c0; ch < c1; ++ch) {
     const int cs = ch * kWideChunk, ce = min(cs + kWideChunk, nnz);
@@ -389,14 +404,16 @@ struct ColVisit {
   int n, ch, lane;
   int ql;            // perm of this lane's key of the current 32-key window
   float4 pcol;       // P row of the current column (this lane's elements)
+  float4 pnext;      // P row of column pnext_c, loaded one column ahead
+  int pnext_c;
   float t[kPairs];   // this lane's parts of the batch's dot products
 
-  __device__ __forceinline__ void begin(int c, int lane_) {
+  __device__ __forceinline__ void begin(int c, int after) {
     if (!perm) return;
-    pcol = ld4(P, c, lane_ & 15);
-    // the next columns' rows of P into L2 (they are loaded at the next switches)
-    if (lane_ < 2 && c + 1 + lane_ < n)
-      prefetch_l2_range(P, (long long)(c + 1 + lane_) * 64, (long long)(c + 2 + lane_) * 64);
+    const int sl = lane & 15;
+    pcol = c == pnext_c ? pnext : ld4(P, c, sl);
+    pnext_c = after;
+    if (after >= 0) pnext = ld4(P, after, sl);
   }
   __device__ __forceinline__ void window(int base, int nk, int lane_) {
     if (perm) ql = lane_ < nk ? __ldg(perm + base + lane_) : 0;
@@ -445,6 +462,8 @@ __global__ void __launch_bounds__(kWideThreads, kWalkCtas)
   vis.lane = lane;
   vis.ql = 0;
   vis.pcol = zero4();
+  vis.pnext = zero4();
+  vis.pnext_c = -1;
 #pragma unroll
   for (int u = 0; u < kPairs; ++u) vis.t[u] = 0.f;
   int hint = 0;

@@ -146,10 +146,21 @@ __global__ void __launch_bounds__(kRowThreads)
         const int t = sub * 4 + grp;
         const int rs = __shfl_sync(FULL_MASK, p0, t), re = __shfl_sync(FULL_MASK, p1, t);
         const float rt = __shfl_sync(FULL_MASK, rr, t);
-        for (int q = rs + gl; q < re; q += kRowLanes) {
-          const int jj = __ldg(cols + q);
-          if (dA) dA[q] = rt * op.gather(jj);
-          if (dxa) atomicAdd(dxa + jj, __ldg(val + q) * rt);
+        if (!dxa) {
+          for (int q = rs + gl; q < re; q += kRowLanes) dA[q] = rt * op.gather(__ldg(cols + q));
+          continue;
+        }
+        // the scatter: every lane runs the longest group's trip count, so the
+        // warp-aggregated atomics see the whole warp (inactive lanes: idx -1)
+        int trips = (re - rs + kRowLanes - 1) / kRowLanes;
+#pragma unroll
+        for (int o = 16; o >= kRowLanes; o >>= 1) trips = max(trips, __shfl_xor_sync(FULL_MASK, trips, o));
+        for (int it = 0; it < trips; ++it) {
+          const int q = rs + gl + it * kRowLanes;
+          const bool act = q < re;
+          const int jj = act ? __ldg(cols + q) : -1;
+          if (dA && act) dA[q] = rt * op.gather(jj);
+          agg_atomic_add(dxa, jj, act ? __ldg(val + q) * rt : 0.f, FULL_MASK);
         }
       }
     }

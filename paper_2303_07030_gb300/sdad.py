@@ -38,7 +38,7 @@ EXPORTS = [
     "sdad_smvm_grad", "sdad_smmm_grad", "sdad_csr_gram_pattern",
     "sdad_batax_grad",
     "sdad_timing_enable", "sdad_timing_reset", "sdad_timing_count", "sdad_timing_get",
-    "sdad_probe_fma", "sdad_gather_by_perm", "sdad_gnn_jvp",
+    "sdad_probe_fma", "sdad_gather_by_perm", "sdad_gnn_jvp", "sdad_lsq_coo_grad",
 ]
 
 
@@ -58,6 +58,13 @@ class sdad_csr(ctypes.Structure):
         ("bcsc_ptr", ctypes.c_void_p), ("bcsc_key", ctypes.c_void_p), ("bcsc_val", ctypes.c_void_p),
         ("bcsc_ncols", ctypes.c_int32), ("bcsc_cols", ctypes.c_void_p),
         ("bcsc_rest_nnz", ctypes.c_int64), ("csc_perm", ctypes.c_void_p),
+    ]
+
+
+class sdad_coo(ctypes.Structure):
+    _fields_ = [
+        ("m", ctypes.c_int32), ("n", ctypes.c_int32), ("nnz", ctypes.c_int64),
+        ("row", ctypes.c_void_p), ("col", ctypes.c_void_p), ("val", ctypes.c_void_p),
     ]
 
 
@@ -124,6 +131,7 @@ def lib():
             "sdad_gather_by_perm": ([vp, i64, vp, i64, vp, vp], i32),
             "sdad_gnn_jvp": ([P(sdad_csr), vp, vp, vp, i32, i32, vp, vp, vp, vp, vp, vp, sz, vp],
                              i32),
+            "sdad_lsq_coo_grad": ([P(sdad_coo), vp, vp, vp, vp, vp, vp, sz, vp], i32),
         }
         for name, (args, res) in sigs.items():
             fn = getattr(L, name)
@@ -525,6 +533,13 @@ def sdad_mf_jvp(R, U, V, k, lam, loss, loss_t, R_t_val=None, U_t=None, V_t=None,
     _check(lib().sdad_mf_jvp(ctypes.byref(d), _ptr(U), _ptr(V), k, float(lam), _ptr(R_t_val),
                              _ptr(U_t), _ptr(V_t), _ptr(loss), _ptr(loss_t), wp, wb,
                              _stream(stream)), "sdad_mf_jvp")
+
+
+def sdad_lsq_coo_grad(A, x, y, loss, dx=None, dA_val=None, ws=None, stream=None):
+    """A: an sdad_coo (device row, col, val in entry order)."""
+    wp, wb = _ws(ws)
+    _check(lib().sdad_lsq_coo_grad(ctypes.byref(A), _ptr(x), _ptr(y), _ptr(loss), _ptr(dx),
+                                   _ptr(dA_val), wp, wb, _stream(stream)), "sdad_lsq_coo_grad")
 
 
 def sdad_gnn_jvp(A, H, W, Z, f_in, f_out, loss, loss_t, A_t_val=None, H_t=None, W_t=None,

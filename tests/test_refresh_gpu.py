@@ -35,7 +35,7 @@ def test_gather_contract():
     perm = rng.integers(-1, 1000, 3001).astype(np.int32)
     perm[::7] = -1
     perm[5] = 1000          # out of range reads as 0 as well
-    out = torch.full((perm.size,), float("nan"), device="cuda")
+    out = torch.full((perm.size,), float("nan"), dtype=torch.float32, device="cuda")
     S.sdad_gather_by_perm(torch.from_numpy(src).cuda(), torch.from_numpy(perm).cuda(), out)
     torch.cuda.synchronize()
     want = np.where((perm >= 0) & (perm < src.size), src[np.clip(perm, 0, src.size - 1)], 0)
