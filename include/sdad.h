@@ -96,7 +96,9 @@ sdad_status sdad_csr_from_coo(int32_t m, int32_t n, int64_t nnz_in, const int32_
                               const int32_t* col, const float* val, int32_t* rowptr,
                               int32_t* colidx, float* val_out, int64_t* nnz_out);
 
-/* CSR pattern -> CSC pattern plus the transpose permutation.
+/* CSR pattern -> CSC pattern plus the transpose permutation (the CSC
+ * storage of Fig. "storage_spec", Sec. 5.3; a second physical format of the
+ * same dictionary).
  *   rowptr[m+1], colidx[nnz] (host, sorted within rows, no duplicates)
  *   colptr      out, host int32[n+1]
  *   rowidx      out, host int32[nnz]; rows ascending within each column
@@ -109,7 +111,9 @@ sdad_status sdad_csr_transpose(int32_t m, int32_t n, int64_t nnz, const int32_t*
                                const int32_t* colidx, int32_t* colptr, int32_t* rowidx,
                                int32_t* perm);
 
-/* Ranking of the columns of a sparse matrix by their number of keys: the
+/* Ranking of the columns of a sparse matrix by their number of keys (a
+ * further physical numbering of the same dictionary, in the spirit of Sec.
+ * 5.3's separation of storage from expression; not in the paper): the
  * columns with most keys get the smallest ranks (equal counts: ascending
  * column).  The ranked ids are an alternative physical column numbering of
  * the same matrix: the key (i, j) at CSR slot p is stored as (i, rank(j)),
@@ -124,7 +128,8 @@ sdad_status sdad_csr_transpose(int32_t m, int32_t n, int64_t nnz, const int32_t*
 sdad_status sdad_csr_rank_columns(int32_t n, int64_t nnz, const int32_t* colidx,
                                   int32_t* rcolidx, int32_t* rankcol);
 
-/* Row-blocked CSC twin of some or all columns: the keys of those columns
+/* Row-blocked CSC twin of some or all columns (a blocked storage of the same
+ * dictionary, Sec. 5.3; not one of the paper's formats): the keys of those columns
  * sorted by (row block, column, row), where a row block is 2^rb_log2
  * consecutive rows.  Each key is packed in 32 bits as
  *   key = (h << rb_log2) | (row - first row of its block),
@@ -160,7 +165,7 @@ sdad_status sdad_csr_block_transpose(int32_t m, int32_t n, int64_t nnz, const in
                                      const int32_t* cols, int32_t* blkptr, uint32_t* bkey,
                                      int32_t* bperm, int64_t* bnnz);
 
-/* CSC twin of the keys whose column is NOT in `cols` (the complement of a
+/* CSC twin (Sec. 5.3) of the keys whose column is NOT in `cols` (the complement of a
  * column-restricted sdad_csr_block_transpose).
  *   rowptr[m+1], colidx[nnz]      host CSR pattern (sorted within rows)
  *   ncols, cols  host int32[ncols], strictly ascending column ids in [0, n)
@@ -175,7 +180,8 @@ sdad_status sdad_csr_transpose_rest(int32_t m, int32_t n, int64_t nnz, const int
                                     int32_t* colptr, int32_t* rowidx, int32_t* perm,
                                     int64_t* rnnz);
 
-/* Mode index of a 3-way COO tensor: a stable sort of the entries by their
+/* Mode index of a 3-way COO tensor (the tensor dictionaries of Sec. 3,
+ * stored as COO, Sec. 5.3): a stable sort of the entries by their
  * mode-`mode` index.
  *   i, j, k     host int32[nnz]; dims[3] the tensor shape
  *   perm        out, host int32[nnz]: entry numbers, grouped by idx_mode,
@@ -271,8 +277,15 @@ typedef struct {
 
 /* How the transposed product (A^T times a dense operand) is formed. */
 typedef enum {
-  SDAD_T_AUTO = 0,    /* library's choice, by measured throughput: CSC for the
-                         CSR losses, ATOMIC for CP (see sdad_cp3_grad)        */
+  SDAD_T_AUTO = 0,    /* library's choice, by measured throughput: where both
+                         modes are possible, the first AUTO call on an operand
+                         (identified by its device, two of its device pointers,
+                         its sizes and the outputs asked for) runs both twice,
+                         times them with events on the call's stream (it waits
+                         for the stream) and keeps the faster; later AUTO calls
+                         run the kept one.  Inside a stream capture no timing
+                         is done: a choice made earlier, else CSC (ATOMIC for
+                         CP).  Where only one mode's arrays are given, that one */
   SDAD_T_CSC = 1,     /* atomic-free column pass over the CSC twin (deterministic) */
   SDAD_T_ATOMIC = 2   /* scattered from the row pass with atomic adds          */
 } sdad_tmode;
@@ -330,7 +343,9 @@ sdad_status sdad_workspace_set_wait_limit(void* ws, int64_t polls, void* stream)
  * Loss + gradient entry points.  All pointers are device pointers.
  * ======================================================================== */
 
-/* Least squares  L = 1/2 ||A x - y||^2   (A: m x n).
+/* Least squares  L = 1/2 ||A x - y||^2   (A: m x n).  One call of
+ * `gradient e x` (Sec. 4.3) for each differentiated operand; the gradient
+ * w.r.t. A lives on keys(A) (Fig. "api"), exact up to rounding (Sec. 6).
  *   x[n], y[m]       inputs (may be NULL when n = 0, resp. m = 0)
  *   loss             out, one double
  *   dx[n]            out, dL/dx = A^T r with r = A x - y       (nullable)
@@ -340,8 +355,9 @@ sdad_status sdad_workspace_set_wait_limit(void* ws, int64_t polls, void* stream)
  * With ranked columns (A->rcolidx, A->rankcol) the row pass reads rcolidx
  * instead of colidx and gathers from a copy of x in ranked order (most used
  * entries first, so they share cache lines); outputs are in the original
- * column order.  SDAD_T_CSC (and AUTO) is bit-reproducible; SDAD_T_ATOMIC
- * adds the transposed product with float atomics (order not fixed).
+ * column order.  SDAD_T_CSC is bit-reproducible; SDAD_T_ATOMIC adds the
+ * transposed product with warp-aggregated float atomics (order not fixed);
+ * AUTO is measured (see sdad_tmode), or ATOMIC without a column structure.
  * Errors: NULL/SHAPE/ALIGN/OVERFLOW/WORKSPACE/CUDA/UNSUPPORTED. */
 sdad_status sdad_lsq_grad(const sdad_csr* A, const float* x, const float* y, double* loss,
                           float* dx, float* dA_val, sdad_tmode tmode, void* ws, size_t ws_bytes,
@@ -360,7 +376,8 @@ sdad_status sdad_lsq_grad(const sdad_csr* A, const float* x, const float* y, dou
 sdad_status sdad_lsq_coo_grad(const sdad_coo* A, const float* x, const float* y, double* loss,
                               float* dx, float* dA_val, void* ws, size_t ws_bytes, void* stream);
 
-/* Logistic regression over m samples (rows of X: m x n), labels y in [0, 1]:
+/* Logistic regression over m samples (rows of X: m x n), labels y in [0, 1]
+ * (gradient on keys as Sec. 4.3 / Fig. "api"; the SMVM-like product of Sec. 7.1):
  *   z = X w,  L = (1/m) sum_i [log(1 + e^{z_i}) - y_i z_i]
  *   dw[n]     out, X^T (sigmoid(z) - y) / m                     (nullable)
  *   dX_val    out, on keys(X) in CSR order: (sigmoid(z_i) - y_i) w_j / m
@@ -370,17 +387,23 @@ sdad_status sdad_logreg_grad(const sdad_csr* X, const float* w, const float* y, 
                              float* dw, float* dX_val, sdad_tmode tmode, void* ws,
                              size_t ws_bytes, void* stream);
 
-/* Matrix factorisation on the observed keys of R (m x n):
+/* Matrix factorisation on the observed keys of R (m x n) (sums over the
+ * dictionary's keys, Sec. 3; dR on keys(R), Sec. 4.3):
  *   L = sum_{(i,j) in keys(R)} (R_ij - U_i . V_j)^2 + lambda (|U|^2 + |V|^2)
  *   U[m x k], V[n x k] inputs; k = 64 in this version
  *   dU[m x k], dV[n x k] out (nullable); dR_val[nnz] out, 2 e_ij in CSR order
- *   (nullable).  dV: SDAD_T_CSC (or AUTO) runs a column pass over R's CSC
- *   twin; SDAD_T_ATOMIC scatters from the row pass with vector atomics. */
+ *   (nullable).  dV: SDAD_T_CSC runs a column pass over R's CSC twin
+ *   (bit-reproducible); SDAD_T_ATOMIC is one pass over the CSR that gathers
+ *   each V row once and scatters dV with vector atomics (with ranked columns,
+ *   rcolidx / rankcol, the 64 most used columns are summed in shared memory
+ *   first; order of additions not fixed); AUTO is measured (see sdad_tmode),
+ *   or ATOMIC when R has no CSC twin. */
 sdad_status sdad_mf_grad(const sdad_csr* R, const float* U, const float* V, int32_t k,
                          float lambda, double* loss, float* dU, float* dV, float* dR_val,
                          sdad_tmode tmode, void* ws, size_t ws_bytes, void* stream);
 
-/* CP decomposition of a 3-way tensor T (dims d0 x d1 x d2, nnz entries):
+/* CP decomposition of a 3-way tensor T (dims d0 x d1 x d2, nnz entries)
+ * (a sum over the tensor dictionary's entries, Sec. 3; dT on its keys, Sec. 4.3):
  *   e_n = T_n - sum_r A_{i r} B_{j r} C_{k r},   L = sum_n e_n^2
  *   A[d0 x R], B[d1 x R], C[d2 x R] inputs; R = 32 in this version
  *   dA, dB, dC out (nullable): dA_i = -2 sum_{n: i_n = i} e_n (B_j * C_k), ...
@@ -390,14 +413,15 @@ sdad_status sdad_mf_grad(const sdad_csr* R, const float* U, const float* V, int3
  *   bit-reproducible.
  *   SDAD_T_ATOMIC: one pass over the entry-order arrays (idx, val) that
  *   scatters all three factor gradients with atomic adds (order not fixed).
- *   SDAD_T_AUTO: ATOMIC when the entry-order arrays are given (measured
- *   faster: half the factor-row gathers), else CSC. */
+ *   SDAD_T_AUTO: measured (see sdad_tmode) when both layouts are given,
+ *   else the one given. */
 sdad_status sdad_cp3_grad(const sdad_coo3* T, const float* A, const float* B, const float* C,
                           int32_t rank, double* loss, float* dA, float* dB, float* dC,
                           float* dT_val, sdad_tmode tmode, void* ws, size_t ws_bytes,
                           void* stream);
 
-/* Graph propagation  Y = A (H W),  L = 1/2 ||Y - Z||^2   (A: m x n graph):
+/* Graph propagation  Y = A (H W),  L = 1/2 ||Y - Z||^2   (A: m x n graph)
+ * (the GNN use case of Sec. 9; dA on keys(A), Sec. 4.3):
  *   H[n x f_in], W[f_in x f_out], Z[m x f_out]; f_in = 128, f_out = 64 here
  *   dA_val[nnz] out, on keys(A): D_i . (H W)_j with D = Y - Z  (nullable)
  *   dH[n x f_in] out, (A^T D) W^T                              (nullable)
@@ -410,7 +434,7 @@ sdad_status sdad_gnn_grad(const sdad_csr* A, const float* H, const float* W, con
                           int32_t f_in, int32_t f_out, double* loss, float* dA_val, float* dH,
                           float* dW, sdad_tmode tmode, void* ws, size_t ws_bytes, void* stream);
 
-/* Forward mode (the tensorized forward-mode rules of Sec. 4 with a real
+/* Forward mode (the tensorized forward-mode rules of Sec. 4.2 with a real
  * tangent): the loss and its directional derivative along a tangent of the
  * inputs, in one pass over A's rows.
  *   x_t[n]        tangent of x (resp. w)                        (nullable: 0)

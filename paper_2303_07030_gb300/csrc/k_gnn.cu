@@ -37,11 +37,18 @@ namespace sdad {
 constexpr int kWideChunk = kMinCap;   // 1024 keys: the piece slots are per kMinCap keys
 constexpr int kWideThreads = 256;
 constexpr int kWideWarps = kWideThreads / 32;
+// Loading the next row's Z (forward walk) or the next column's P row (column
+// walk) one segment ahead measured neutral to slightly slower on the R-MAT
+// graph (registers); kept as an option.
 #ifndef SDAD_WALK_LOOKAHEAD
-#define SDAD_WALK_LOOKAHEAD 1
+#define SDAD_WALK_LOOKAHEAD 0
 #endif
-constexpr bool kWalkLookahead = SDAD_WALK_LOOKAHEAD;   // next row's Z / next column's P loaded ahead
-constexpr int kWalkCtas = 3;          // resident CTAs per SM the walks are compiled for (<= 85 registers)
+constexpr bool kWalkLookahead = SDAD_WALK_LOOKAHEAD;
+// Resident CTAs per SM the walks are compiled for: the forward walk measured
+// fastest at 4 (64 registers), the column walk (which also holds P_c and the
+// batch's dot products) at 3.
+constexpr int kFwdCtas = 4;
+constexpr int kColCtas = 3;
 
 __device__ __forceinline__ float2 ld2(const float* base, int r, int lane) {
   return __ldg(reinterpret_cast<const float2*>(base + (size_t)r * 64) + lane);
@@ -69,8 +76,8 @@ __device__ __forceinline__ Seg next_segment(const int32_t* __restrict__ ptr, int
     const int s1 = __shfl_sync(FULL_MASK, pv, f);
     const int before = __shfl_sync(FULL_MASK, pv, (f + 31) & 31);
     // the segment holding key s1: the last i with ptr[i] <= s1
-    const unsigned b2 = __ballot_sync(FULL_MASK, pv > s1 && pv != INT_MAX);
-    const int after = (kWalkLookahead && b2) ? lo + __ffs(b2) - 1 : -1;
+    const unsigned b2 = kWalkLookahead ? __ballot_sync(FULL_MASK, pv > s1 && pv != INT_MAX) : 0u;
+    const int after = b2 ? lo + __ffs(b2) - 1 : -1;
     // f = 0 would mean p lies in segment lo itself (not so where the walks call this)
     return Seg{lo + f, f ? before : __ldg(ptr + lo), s1, after};
   }
@@ -217,6 +224,7 @@ struct FwdVisit {
   int znext_r;
 
   __device__ __forceinline__ void begin(int r, int after) {
+    if (!kWalkLookahead) return;   // Z is then read when the row ends
     const int sl = lane & 15;
     zr = r == znext_r ? znext : ld4(Z, r, sl);
     znext_r = after;
@@ -229,6 +237,7 @@ struct FwdVisit {
   __device__ __forceinline__ void segment(int r, int s0, int s1, float4 tot, int cs, int ce) {
     if (pc.cut(ch, r, s0, s1, cs, ce, tot, lane)) return;
     const int sl = lane & 15;
+    if (!kWalkLookahead) zr = ld4(Z, r, sl);
     const float4 d = make_float4(tot.x - zr.x, tot.y - zr.y, tot.z - zr.z, tot.w - zr.w);
     if (lane < 16) {
       st4(D, r, sl, d);
@@ -242,7 +251,7 @@ struct FwdVisit {
 // permutation lets the column walk compute it); a template parameter so that
 // the plain walk does not carry the SDDMM's registers.
 template <bool WITH_DA>
-__global__ void __launch_bounds__(kWideThreads, kWalkCtas)
+__global__ void __launch_bounds__(kWideThreads, kFwdCtas)
     gnn_fwd_kernel(const int32_t* __restrict__ rowptr, const int32_t* __restrict__ colidx,
                    const float* __restrict__ val, int m, int nnz, int nchunks,
                    const float* __restrict__ P, const float* __restrict__ Z, float* __restrict__ D,
@@ -411,6 +420,10 @@ struct ColVisit {
   __device__ __forceinline__ void begin(int c, int after) {
     if (!perm) return;
     const int sl = lane & 15;
+    if (!kWalkLookahead) {
+      pcol = ld4(P, c, sl);
+      return;
+    }
     pcol = c == pnext_c ? pnext : ld4(P, c, sl);
     pnext_c = after;
     if (after >= 0) pnext = ld4(P, after, sl);
@@ -442,7 +455,7 @@ struct ColVisit {
 };
 
 // perm != NULL: also dA on the keys
-__global__ void __launch_bounds__(kWideThreads, kWalkCtas)
+__global__ void __launch_bounds__(kWideThreads, kColCtas)
     gnn_col_kernel(const int32_t* __restrict__ colptr, const int32_t* __restrict__ rowidx,
                    const float* __restrict__ val_csc, int n, int nnz, int nchunks,
                    const float* __restrict__ D, float* __restrict__ G, ChunkPieces pc,
