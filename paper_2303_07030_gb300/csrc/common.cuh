@@ -23,7 +23,8 @@ struct WsHeader {
   int32_t status;       // sticky error code (0 = ok), cleared by sdad_check
   uint32_t ticket;      // last-CTA ticket of the loss reduction, back to 0 after use
   uint32_t wait_polls;  // 0: bounded waits poll kWaitPolls times; v > 0: v - 1 times
-  uint32_t pad[61];
+  uint32_t work[2];     // work counters of the graph walks (chunk groups handed out)
+  uint32_t pad[59];
 };
 static_assert(sizeof(WsHeader) == 256, "header is 256 bytes");
 

@@ -11,19 +11,21 @@
 // as hi*hi' + hi*lo' + lo*hi' (three kind::f16 MMAs, fp32 accumulation in
 // tensor memory): about 2^-15 relative error per product, well inside the
 // 1e-4 normwise gradient tolerance (4e-6 normwise for P on the workload's
-// distributions).  BF16 parts take half the shared memory of TF32 parts, so a
-// CTA holds two tiles and W, and the MMAs issue at the BF16 rate.
+// distributions).  No tensor-memory accumulation runs longer than one tile:
+// the tiles' dW are added in fp32 registers.
 //
-// Pipeline (one CTA of 16 warps per SM, 128-row tiles t = blockIdx.x + i *
-// gridDim.x): the threads load tile i+1 into registers (16-byte streaming
-// loads) while the tensor cores work on tile i and the threads drain tile
-// i-1's accumulator from tensor memory (tcgen05.ld) to global memory.  The
-// next tile is split and written into the other of two shared-memory buffers
-// in the 128-byte swizzled layout, and thread 0 issues its MMAs; each tile's
-// MMAs commit to the mbarrier of its buffer, which frees the buffer and
-// publishes the accumulator.  Accumulators are double-buffered in tensor
-// memory.  Every wait is bounded; a kernel that gives up still waits for the
-// MMAs it issued before it frees tensor memory.
+// Pipeline (one CTA of 16 warps per SM, persistent over 128-row tiles t =
+// blockIdx.x + i * gridDim.x; a tile's rows are one contiguous block of H
+// and of G): thread 0 streams each tile into shared memory with bulk copies
+// (cp.async.bulk, completion counted in bytes on an mbarrier), two 64-row
+// halves at a time in a ring of two raw stages; the threads split a landed
+// half into BF16 hi and lo parts, written in the 128-byte swizzled layout the
+// MMAs read, and the freed stage is refilled with the next tile's half at
+// once.  Thread 0 issues the tile's MMAs, which commit to an mbarrier; while
+// the tensor cores work, the threads drain the previous tile's accumulator
+// (tcgen05.ld) to global memory (accumulators are double-buffered in tensor
+// memory).  Every wait is bounded; a kernel that gives up still waits for
+// the copies and MMAs it issued before it leaves.
 //
 // Operand layouts (all 128-byte swizzled; a "block" is a stack of 128-byte
 // rows, each row 64 BF16 values):
@@ -47,21 +49,28 @@ namespace sdad {
 
 constexpr int kFin = 128, kFout = 64;
 constexpr int kTileM = 128;
+constexpr int kHalfM = 64;              // rows per raw stage
 constexpr int kDenseThreads = 512;
-constexpr uint32_t kBlk = 128 * 128;   // bytes of a 128-row block
+constexpr uint32_t kBlk = 128 * 128;    // bytes of a 128-row block of 128-byte rows
+constexpr uint32_t kHRow = kFin * 4;    // bytes of an fp32 row of H
+constexpr uint32_t kGRow = kFout * 4;   // ... of G
 
 // shared-memory map of proj_fwd_kernel (from a 1024-byte aligned base)
-constexpr uint32_t kFwdA = 0;                          // [buf][hi|lo][kb] x kBlk
-constexpr uint32_t kFwdW = kFwdA + 8 * kBlk;           // W^T: [hi|lo][kb] x 64 rows x 128 B
+constexpr uint32_t kFwdRaw = 0;                         // 2 stages x 64 rows of H (fp32)
+constexpr uint32_t kFwdRawStage = kHalfM * kHRow;       // 32 KB
+constexpr uint32_t kFwdA = kFwdRaw + 2 * kFwdRawStage;  // [hi|lo][kb] x kBlk
+constexpr uint32_t kFwdW = kFwdA + 4 * kBlk;            // W^T: [hi|lo][kb] x 64 rows x 128 B
 constexpr uint32_t kFwdBar = kFwdW + 4 * 64 * 128;
-constexpr uint32_t kFwdSmem = kFwdBar + 32 + 1024;     // two barriers, the TMEM slot, alignment
+constexpr uint32_t kFwdSmem = kFwdBar + 64 + 1024;      // barriers, the TMEM slot, alignment
 // shared-memory map of proj_bwd_kernel
-constexpr uint32_t kBwdG = 0;                          // [buf][hi|lo] x kBlk
-constexpr uint32_t kBwdH = kBwdG + 4 * kBlk;           // [buf][hi|lo][block] x kBlk
-constexpr uint32_t kBwdW = kBwdH + 8 * kBlk;           // W: [hi|lo] x kBlk
+constexpr uint32_t kBwdRawStage = kHalfM * (kHRow + kGRow);   // 48 KB: 64 rows of H, then of G
+constexpr uint32_t kBwdRaw = 0;
+constexpr uint32_t kBwdG = kBwdRaw + 2 * kBwdRawStage;  // [hi|lo] x kBlk
+constexpr uint32_t kBwdH = kBwdG + 2 * kBlk;            // [hi|lo][block] x kBlk
+constexpr uint32_t kBwdW = kBwdH + 4 * kBlk;            // W: [hi|lo] x kBlk
 constexpr uint32_t kBwdBar = kBwdW + 2 * kBlk;
-constexpr uint32_t kBwdSmem = kBwdBar + 32 + 1024;
-static_assert(kBwdSmem <= 227 * 1024, "shared memory of one CTA");
+constexpr uint32_t kBwdSmem = kBwdBar + 64 + 1024;
+static_assert(kFwdSmem <= 227 * 1024 && kBwdSmem <= 227 * 1024, "shared memory of one CTA");
 
 __device__ __forceinline__ uint32_t bf2_bits(__nv_bfloat162 v) {
   return *reinterpret_cast<const uint32_t*>(&v);
@@ -83,6 +92,14 @@ __device__ __forceinline__ void sts64(uint32_t addr, uint2 v) {
 __device__ __forceinline__ void sts16(uint32_t addr, uint16_t v) {
   asm volatile("st.shared.b16 [%0], %1;" ::"r"(addr), "h"(v) : "memory");
 }
+__device__ __forceinline__ float4 lds128(uint32_t addr) {
+  float4 v;
+  asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(addr)
+               : "memory");
+  return v;
+}
 
 // writes the hi and lo parts of one fp32 value at byte offset `off` of the
 // hi and lo copies
@@ -95,33 +112,35 @@ __device__ __forceinline__ void put1(uint32_t hi_base, uint32_t lo_base, uint32_
 
 __device__ __forceinline__ uint32_t align1024(uint32_t a) { return (a + 1023u) & ~1023u; }
 
-// 16-byte loads of one 128-row tile of a row-major [n x (C4 * 4)] fp32 matrix
-// (rows past n read as zero): element j of this thread is float4 q = tid +
-// kDenseThreads * j, at row q / C4, column 4 (q % C4).
-template <int C4, int NJ>
-__device__ __forceinline__ void load_tile(float4 (&R)[NJ], const float* __restrict__ X, int row0,
-                                          int n) {
-#pragma unroll
-  for (int j = 0; j < NJ; ++j) {
-    const int q = threadIdx.x + kDenseThreads * j;
-    const int r = row0 + q / C4;
-    R[j] = r < n ? __ldcs(reinterpret_cast<const float4*>(X + (size_t)r * (C4 * 4)) + (q % C4))
-                 : make_float4(0.f, 0.f, 0.f, 0.f);
-  }
+// bulk copy of `bytes` (a multiple of 16) from global memory to the shared
+// address `dst`, completion counted on the mbarrier at shared address `bar`
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes,
+                                          uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
+          "r"(dst),
+      "l"(src), "r"(bytes), "r"(bar)
+      : "memory");
 }
 
-// ... and their hi / lo parts into the swizzled blocks at hi_base / lo_base
-// (block b holds columns 64 b .. 64 b + 63; blocks kBlk bytes apart)
-template <int C4, int NJ>
-__device__ __forceinline__ void store_tile(const float4 (&R)[NJ], uint32_t hi_base,
-                                           uint32_t lo_base) {
+// rows of [r0, r0 + 64) that exist (r0 < n gives at least one)
+__device__ __forceinline__ int half_rows(int r0, int n) { return max(0, min(kHalfM, n - r0)); }
+
+// Splits 64 landed rows of fp32 data (row-major, C4 float4 per row, at raw
+// address `raw`) into the hi / lo swizzled blocks (block b holds columns
+// 64 b .. 64 b + 63, blocks kBlk apart), at tile rows row0 .. row0 + 63.
+// Rows at or past `valid` read as zero.
+template <int C4>
+__device__ __forceinline__ void split_half(uint32_t raw, uint32_t hi_base, uint32_t lo_base,
+                                           int row0, int valid) {
+  constexpr int kN = kHalfM * C4;   // float4 of the half
 #pragma unroll
-  for (int j = 0; j < NJ; ++j) {
-    const int q = threadIdx.x + kDenseThreads * j;
+  for (int q = threadIdx.x; q < kN; q += kDenseThreads) {
     const int r = q / C4, f = 4 * (q % C4);
-    const uint32_t off = (uint32_t)(f >> 6) * kBlk + tc::sw128_offset_b16(r, f & 63);
+    const float4 x = r < valid ? lds128(raw + 16u * (uint32_t)q) : make_float4(0.f, 0.f, 0.f, 0.f);
+    const uint32_t off = (uint32_t)(f >> 6) * kBlk + tc::sw128_offset_b16(row0 + r, f & 63);
     uint2 hi, lo;
-    split4(R[j], hi, lo);
+    split4(x, hi, lo);
     sts64(hi_base + off, hi);
     sts64(lo_base + off, lo);
   }
@@ -136,8 +155,8 @@ __device__ __forceinline__ uint64_t mndesc(uint32_t block, int s) {
   return tc::smem_desc_sw128_mn(block + 2048u * (uint32_t)s, kBlk);
 }
 
-// drains COLS accumulator columns (starting at column c0 of the tile's
-// accumulator) for this warp's 32 rows into out rows of width OUTW
+// drains COLS accumulator columns for this warp's 32 rows into out rows of
+// width OUTW (rows at or past n are not stored)
 template <int COLS, bool STREAM>
 __device__ __forceinline__ void drain_rows(uint32_t taddr, float* __restrict__ out, int OUTW,
                                            int row, int col, int n) {
@@ -156,6 +175,20 @@ __device__ __forceinline__ void drain_rows(uint32_t taddr, float* __restrict__ o
   }
 }
 
+// The raw-stage ring shared by both kernels: stage h (0, 1) holds half h of
+// a tile; n_issued / n_waited count the uses of each stage's barrier.
+struct RawRing {
+  uint64_t* full;   // two mbarriers
+  int n_issued[2];
+  int n_waited[2];
+  __device__ __forceinline__ uint32_t parity(int h) const { return (uint32_t)(n_waited[h] & 1); }
+  // before leaving: wait for every copy issued but not waited for
+  __device__ __forceinline__ void drain(WsHeader* hdr) {
+    for (int h = 0; h < 2; ++h)
+      if (n_issued[h] > n_waited[h]) mbar_drain(&full[h], (uint32_t)((n_issued[h] - 1) & 1), hdr);
+  }
+};
+
 // ---------------------------------------------------------------------------
 // P = H W
 // ---------------------------------------------------------------------------
@@ -165,30 +198,37 @@ __global__ void __launch_bounds__(kDenseThreads, 1)
   extern __shared__ unsigned char dense_smem[];
   const uint32_t base = align1024(smem_u32(dense_smem));
   unsigned char* gbase = dense_smem + (base - smem_u32(dense_smem));
-  uint64_t* bar = reinterpret_cast<uint64_t*>(gbase + kFwdBar);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + kFwdBar + 16);
+  uint64_t* full = reinterpret_cast<uint64_t*>(gbase + kFwdBar);
+  uint64_t* mma = full + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + kFwdBar + 24);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   constexpr uint32_t idesc = tc::idesc_bf16(kTileM, kFout, false, false);
-  auto A = [&](int b, int part, int kb) { return base + kFwdA + (uint32_t)((b * 2 + part) * 2 + kb) * kBlk; };
+  auto A = [&](int part, int kb) { return base + kFwdA + (uint32_t)(part * 2 + kb) * kBlk; };
   auto Wt = [&](int part, int kb) { return base + kFwdW + (uint32_t)(part * 2 + kb) * (64 * 128); };
+  auto raw = [&](int h) { return base + kFwdRaw + (uint32_t)h * kFwdRawStage; };
 
   const int ntiles = (n + kTileM - 1) / kTileM;
   const int grid = gridDim.x;
-  int t = blockIdx.x;
-  float4 R[8];   // the next H tile: 128 rows x 32 float4
-  if (t < ntiles) load_tile<32, 8>(R, H, t * kTileM, n);
-
+  const int nloc = (ntiles - (int)blockIdx.x + grid - 1) / grid;   // >= 1: grid <= tiles
+  RawRing ring{full, {0, 0}, {0, 0}};
   if (tid == 0) {
-    mbar_init(&bar[0], 1);
-    mbar_init(&bar[1], 1);
+    mbar_init(&full[0], 1);
+    mbar_init(&full[1], 1);
+    mbar_init(mma, 1);
     fence_mbar_init();
+    for (int h = 0; h < 2; ++h) {   // tile 0's halves
+      const int r0 = (int)blockIdx.x * kTileM + h * kHalfM;
+      const uint32_t bytes = (uint32_t)half_rows(r0, n) * kHRow;
+      mbar_arrive_expect_tx(&full[h], bytes);
+      if (bytes) bulk_load(raw(h), H + (size_t)r0 * kFin, bytes, smem_u32(&full[h]));
+    }
   }
+  ring.n_issued[0] = ring.n_issued[1] = 1;
   if (warp == 0) tc::tmem_alloc(tmem_slot, 2 * kFout);   // two accumulators of 64 columns
   // operand B = W^T (row n' = column n' of W), once per CTA
   for (int idx = tid; idx < kFin * kFout; idx += kDenseThreads) {
     const int k = idx / kFout, nn = idx % kFout;
-    const uint32_t off = tc::sw128_offset_b16(nn, k & 63);
-    put1(Wt(0, k >> 6), Wt(1, k >> 6), off, __ldg(W + idx));
+    put1(Wt(0, k >> 6), Wt(1, k >> 6), tc::sw128_offset_b16(nn, k & 63), __ldg(W + idx));
   }
   tc::fence_proxy_async_smem();
   tc::fence_before_sync();
@@ -199,54 +239,68 @@ __global__ void __launch_bounds__(kDenseThreads, 1)
   const int q4 = warp & 3, cg = warp >> 2;   // epilogue: TMEM lanes 32 q4.., columns 16 cg..
   bool ok = true;
   int last = -1;   // local index of the last tile whose MMAs were issued
-  int i = 0;
-  for (; t < ntiles; ++i, t += grid) {
-    const int b = i & 1;
-    if (i >= 2) {   // buffer b is free once tile i-2's MMAs are done
-      ok = __syncthreads_and(mbar_wait(&bar[b], ((i >> 1) - 1) & 1, hdr));
+  for (int i = 0; i < nloc; ++i) {
+    const int t = (int)blockIdx.x + i * grid, row0 = t * kTileM;
+    if (i >= 1) {   // the split parts are free once tile i-1's MMAs are done
+      ok = __syncthreads_and(mbar_wait(mma, (uint32_t)((i - 1) & 1), hdr));
       if (!ok) break;
+      tc::fence_after_sync();
     }
-    store_tile<32, 8>(R, A(b, 0, 0), A(b, 1, 0));
-    if (t + grid < ntiles) load_tile<32, 8>(R, H, (t + grid) * kTileM, n);
+    for (int h = 0; h < 2; ++h) {
+      ok = __syncthreads_and(mbar_wait(&full[h], ring.parity(h), hdr));
+      if (!ok) break;
+      ++ring.n_waited[h];
+      split_half<32>(raw(h), A(0, 0), A(1, 0), h * kHalfM, half_rows(row0 + h * kHalfM, n));
+      __syncthreads();   // the stage is read: refill it with the next tile's half
+      if (i + 1 < nloc) {
+        if (tid == 0) {
+          const int r0 = row0 + grid * kTileM + h * kHalfM;
+          const uint32_t bytes = (uint32_t)half_rows(r0, n) * kHRow;
+          mbar_arrive_expect_tx(&full[h], bytes);
+          if (bytes) bulk_load(raw(h), H + (size_t)r0 * kFin, bytes, smem_u32(&full[h]));
+        }
+        ++ring.n_issued[h];
+      }
+    }
+    if (!ok) break;
     tc::fence_proxy_async_smem();
     tc::fence_before_sync();
     __syncthreads();
     if (tid == 0) {
       tc::fence_after_sync();
-      const uint32_t d = tmem + (uint32_t)(kFout * b);
+      const uint32_t d = tmem + (uint32_t)(kFout * (i & 1));
 #pragma unroll
       for (int kb = 0; kb < 2; ++kb)
 #pragma unroll
         for (int s = 0; s < 4; ++s) {
-          const uint64_t ah = kdesc(A(b, 0, kb), s), al = kdesc(A(b, 1, kb), s);
+          const uint64_t ah = kdesc(A(0, kb), s), al = kdesc(A(1, kb), s);
           const uint64_t bh = kdesc(Wt(0, kb), s), bl = kdesc(Wt(1, kb), s);
           tc::mma_bf16(d, ah, bh, idesc, (kb | s) != 0);
           tc::mma_bf16(d, ah, bl, idesc, true);
           tc::mma_bf16(d, al, bh, idesc, true);
         }
-      tc::mma_commit(&bar[b]);
+      tc::mma_commit(mma);
     }
     last = i;
     if (i >= 1) {   // tile i-1's accumulator to P while the tensor cores work on tile i
-      ok = __syncthreads_and(mbar_wait(&bar[b ^ 1], ((i - 1) >> 1) & 1, hdr));
-      if (!ok) break;
-      tc::fence_after_sync();
       const int row = (t - grid) * kTileM + 32 * q4 + lane;
-      drain_rows<16, false>(tmem + ((uint32_t)(32 * q4) << 16) + (uint32_t)(kFout * (b ^ 1) + 16 * cg),
+      drain_rows<16, false>(tmem + ((uint32_t)(32 * q4) << 16) + (uint32_t)(kFout * ((i - 1) & 1) + 16 * cg),
                             P, kFout, row, 16 * cg, n);
     }
   }
   if (ok && last >= 0) {
-    ok = __syncthreads_and(mbar_wait(&bar[last & 1], (last >> 1) & 1, hdr));
+    ok = __syncthreads_and(mbar_wait(mma, (uint32_t)(last & 1), hdr));
     if (ok) {
       tc::fence_after_sync();
-      const int row = (blockIdx.x + last * grid) * kTileM + 32 * q4 + lane;
+      const int row = ((int)blockIdx.x + last * grid) * kTileM + 32 * q4 + lane;
       drain_rows<16, false>(tmem + ((uint32_t)(32 * q4) << 16) + (uint32_t)(kFout * (last & 1) + 16 * cg),
                             P, kFout, row, 16 * cg, n);
     }
   }
-  // a wait gave up: the issued MMAs still write tensor memory; let them end
-  if (!ok && last >= 0) mbar_drain(&bar[last & 1], (last >> 1) & 1, hdr);
+  if (!ok) {   // a wait gave up: let the issued copies land and the MMAs end
+    if (last >= 0) mbar_drain(mma, (uint32_t)(last & 1), hdr);
+    ring.drain(hdr);
+  }
   tc::fence_before_sync();
   __syncthreads();
   if (warp == 0) tc::tmem_dealloc(tmem, 2 * kFout);
@@ -262,34 +316,44 @@ __global__ void __launch_bounds__(kDenseThreads, 1)
   extern __shared__ unsigned char dense_smem[];
   const uint32_t base = align1024(smem_u32(dense_smem));
   unsigned char* gbase = dense_smem + (base - smem_u32(dense_smem));
-  uint64_t* bar = reinterpret_cast<uint64_t*>(gbase + kBwdBar);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + kBwdBar + 16);
+  uint64_t* full = reinterpret_cast<uint64_t*>(gbase + kBwdBar);
+  uint64_t* mma = full + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + kBwdBar + 24);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   constexpr uint32_t idesc_dh = tc::idesc_bf16(kTileM, kFin, false, false);
   constexpr uint32_t idesc_dw = tc::idesc_bf16(kFin, kFout, true, true);
-  // dW of each tile in tensor memory (two accumulators after the two of dH);
-  // the tiles' dW are added in registers in fp32 (each thread 16 entries), so
-  // no tensor-memory accumulation runs longer than one tile's 8 k-steps
+  // tensor memory: two dH accumulators (128 columns each), then two of dW
+  // (64 each); a tile's dW is added in fp32 registers (each thread 16 entries)
   constexpr uint32_t kDwCol = 2 * kFin;
-  auto Gs = [&](int b, int part) { return base + kBwdG + (uint32_t)(b * 2 + part) * kBlk; };
-  auto Hs = [&](int b, int part) { return base + kBwdH + (uint32_t)((b * 2 + part) * 2) * kBlk; };
+  auto Gs = [&](int part) { return base + kBwdG + (uint32_t)part * kBlk; };
+  auto Hs = [&](int part) { return base + kBwdH + (uint32_t)(part * 2) * kBlk; };
   auto Ws = [&](int part) { return base + kBwdW + (uint32_t)part * kBlk; };
+  auto raw = [&](int h) { return base + kBwdRaw + (uint32_t)h * kBwdRawStage; };
+  // thread 0: the copies of rows [r0, r0 + 64) of H and G into stage h
+  auto issue = [&](int h, int r0) {
+    const int rows = half_rows(r0, n);
+    mbar_arrive_expect_tx(&full[h], (uint32_t)rows * (kHRow + kGRow));
+    if (rows) {
+      bulk_load(raw(h), H + (size_t)r0 * kFin, (uint32_t)rows * kHRow, smem_u32(&full[h]));
+      bulk_load(raw(h) + kHalfM * kHRow, G + (size_t)r0 * kFout, (uint32_t)rows * kGRow,
+                smem_u32(&full[h]));
+    }
+  };
 
   const int ntiles = (n + kTileM - 1) / kTileM;
   const int grid = gridDim.x;
-  int t = blockIdx.x;
-  float4 RG[4], RH[8];   // the next tile: G 128 x 16 float4, H 128 x 32 float4
-  if (t < ntiles) {
-    load_tile<16, 4>(RG, G, t * kTileM, n);
-    load_tile<32, 8>(RH, H, t * kTileM, n);
-  }
-
+  const int nloc = (ntiles - (int)blockIdx.x + grid - 1) / grid;   // >= 1: grid <= tiles
+  RawRing ring{full, {0, 0}, {0, 0}};
   if (tid == 0) {
-    mbar_init(&bar[0], 1);
-    mbar_init(&bar[1], 1);
+    mbar_init(&full[0], 1);
+    mbar_init(&full[1], 1);
+    mbar_init(mma, 1);
     fence_mbar_init();
+    issue(0, (int)blockIdx.x * kTileM);
+    issue(1, (int)blockIdx.x * kTileM + kHalfM);
   }
-  if (warp == 0) tc::tmem_alloc(tmem_slot, 512);   // dH: 2 x 128 columns; dW: 2 x 64
+  ring.n_issued[0] = ring.n_issued[1] = 1;
+  if (warp == 0) tc::tmem_alloc(tmem_slot, 512);
   // operand B of dH = W (row n' = row n' of W), once per CTA
   for (int idx = tid; idx < kFin * kFout; idx += kDenseThreads) {
     const int nn = idx / kFout, k = idx % kFout;
@@ -305,77 +369,76 @@ __global__ void __launch_bounds__(kDenseThreads, 1)
   float dwacc[16];   // this thread's entries of the CTA's dW: row 32 q4 + lane, columns 16 cg ..
 #pragma unroll
   for (int c = 0; c < 16; ++c) dwacc[c] = 0.f;
-  // adds tile-buffer bb's dW accumulator to dwacc
-  auto add_dw = [&](int bb) {
+  // tile j's dH to memory (row0: its first row) and its dW into dwacc
+  auto epilogue = [&](int j, int row0) {
+    const uint32_t lanes = (uint32_t)(32 * q4) << 16;
+    if (dH)
+      drain_rows<32, true>(tmem + lanes + (uint32_t)(kFin * (j & 1) + 32 * cg), dH, kFin,
+                           row0 + 32 * q4 + lane, 32 * cg, n);
     float v[16];
-    tc::tmem_ld16(tmem + ((uint32_t)(32 * q4) << 16) + kDwCol + (uint32_t)(kFout * bb + 16 * cg), v);
+    tc::tmem_ld16(tmem + lanes + kDwCol + (uint32_t)(kFout * (j & 1) + 16 * cg), v);
     tc::tmem_wait_ld();
 #pragma unroll
     for (int c = 0; c < 16; ++c) dwacc[c] += v[c];
   };
   bool ok = true;
   int last = -1;
-  int i = 0;
-  for (; t < ntiles; ++i, t += grid) {
-    const int b = i & 1;
-    if (i >= 2) {
-      ok = __syncthreads_and(mbar_wait(&bar[b], ((i >> 1) - 1) & 1, hdr));
+  for (int i = 0; i < nloc; ++i) {
+    const int t = (int)blockIdx.x + i * grid, row0 = t * kTileM;
+    if (i >= 1) {   // the split parts are free once tile i-1's MMAs are done
+      ok = __syncthreads_and(mbar_wait(mma, (uint32_t)((i - 1) & 1), hdr));
       if (!ok) break;
+      tc::fence_after_sync();
     }
-    store_tile<16, 4>(RG, Gs(b, 0), Gs(b, 1));
-    store_tile<32, 8>(RH, Hs(b, 0), Hs(b, 1));
-    if (t + grid < ntiles) {
-      load_tile<16, 4>(RG, G, (t + grid) * kTileM, n);
-      load_tile<32, 8>(RH, H, (t + grid) * kTileM, n);
+    for (int h = 0; h < 2; ++h) {
+      ok = __syncthreads_and(mbar_wait(&full[h], ring.parity(h), hdr));
+      if (!ok) break;
+      ++ring.n_waited[h];
+      const int valid = half_rows(row0 + h * kHalfM, n);
+      split_half<32>(raw(h), Hs(0), Hs(1), h * kHalfM, valid);
+      split_half<16>(raw(h) + kHalfM * kHRow, Gs(0), Gs(1), h * kHalfM, valid);
+      __syncthreads();   // the stage is read: refill it with the next tile's half
+      if (i + 1 < nloc) {
+        if (tid == 0) issue(h, row0 + grid * kTileM + h * kHalfM);
+        ++ring.n_issued[h];
+      }
     }
+    if (!ok) break;
     tc::fence_proxy_async_smem();
     tc::fence_before_sync();
     __syncthreads();
     if (tid == 0) {
       tc::fence_after_sync();
-      // dW += H^T G: M = f_in (MN-major H), N = f_out (MN-major G), K = the tile's rows
+      // dW of the tile: M = f_in (MN-major H), N = f_out (MN-major G), K = the tile's rows
+      const uint32_t dw = tmem + kDwCol + (uint32_t)(kFout * (i & 1));
 #pragma unroll
       for (int s = 0; s < kTileM / 16; ++s) {
-        const uint64_t ah = mndesc(Hs(b, 0), s), al = mndesc(Hs(b, 1), s);
-        const uint64_t bh = mndesc(Gs(b, 0), s), bl = mndesc(Gs(b, 1), s);
-        const uint32_t dw = tmem + kDwCol + (uint32_t)(kFout * b);
+        const uint64_t ah = mndesc(Hs(0), s), al = mndesc(Hs(1), s);
+        const uint64_t bh = mndesc(Gs(0), s), bl = mndesc(Gs(1), s);
         tc::mma_bf16(dw, ah, bh, idesc_dw, s > 0);
         tc::mma_bf16(dw, ah, bl, idesc_dw, true);
         tc::mma_bf16(dw, al, bh, idesc_dw, true);
       }
       // dH = G W^T: M = rows, N = f_in, K = f_out (both K-major)
-      const uint32_t d = tmem + (uint32_t)(kFin * b);
+      const uint32_t d = tmem + (uint32_t)(kFin * (i & 1));
 #pragma unroll
       for (int s = 0; s < (dH ? kFout / 16 : 0); ++s) {
-        const uint64_t ah = kdesc(Gs(b, 0), s), al = kdesc(Gs(b, 1), s);
+        const uint64_t ah = kdesc(Gs(0), s), al = kdesc(Gs(1), s);
         const uint64_t bh = kdesc(Ws(0), s), bl = kdesc(Ws(1), s);
         tc::mma_bf16(d, ah, bh, idesc_dh, s > 0);
         tc::mma_bf16(d, ah, bl, idesc_dh, true);
         tc::mma_bf16(d, al, bh, idesc_dh, true);
       }
-      tc::mma_commit(&bar[b]);
+      tc::mma_commit(mma);
     }
     last = i;
-    if (i >= 1) {   // tile i-1's dH to memory and its dW into dwacc
-      ok = __syncthreads_and(mbar_wait(&bar[b ^ 1], ((i - 1) >> 1) & 1, hdr));
-      if (!ok) break;
-      tc::fence_after_sync();
-      const int row = (t - grid) * kTileM + 32 * q4 + lane;
-      if (dH)
-        drain_rows<32, true>(tmem + ((uint32_t)(32 * q4) << 16) + (uint32_t)(kFin * (b ^ 1) + 32 * cg),
-                             dH, kFin, row, 32 * cg, n);
-      add_dw(b ^ 1);
-    }
+    if (i >= 1) epilogue(i - 1, (t - grid) * kTileM);   // while the tensor cores work on tile i
   }
   if (ok && last >= 0) {
-    ok = __syncthreads_and(mbar_wait(&bar[last & 1], (last >> 1) & 1, hdr));
+    ok = __syncthreads_and(mbar_wait(mma, (uint32_t)(last & 1), hdr));
     if (ok) {
       tc::fence_after_sync();
-      const int row = (blockIdx.x + last * grid) * kTileM + 32 * q4 + lane;
-      if (dH)
-        drain_rows<32, true>(tmem + ((uint32_t)(32 * q4) << 16) + (uint32_t)(kFin * (last & 1) + 32 * cg),
-                             dH, kFin, row, 32 * cg, n);
-      add_dw(last & 1);
+      epilogue(last, ((int)blockIdx.x + last * grid) * kTileM);
       // this CTA's dW: TMEM lane = f_in, column = f_out
       float4* dst = reinterpret_cast<float4*>(dWpart + (size_t)blockIdx.x * kFin * kFout +
                                               (size_t)(32 * q4 + lane) * kFout + 16 * cg);
@@ -384,7 +447,10 @@ __global__ void __launch_bounds__(kDenseThreads, 1)
         dst[q] = make_float4(dwacc[4 * q], dwacc[4 * q + 1], dwacc[4 * q + 2], dwacc[4 * q + 3]);
     }
   }
-  if (!ok && last >= 0) mbar_drain(&bar[last & 1], (last >> 1) & 1, hdr);
+  if (!ok) {   // a wait gave up: let the issued copies land and the MMAs end
+    if (last >= 0) mbar_drain(mma, (uint32_t)(last & 1), hdr);
+    ring.drain(hdr);
+  }
   tc::fence_before_sync();
   __syncthreads();
   if (warp == 0) tc::tmem_dealloc(tmem, 512);

@@ -85,6 +85,18 @@ __device__ __forceinline__ Seg next_segment(const int32_t* __restrict__ ptr, int
   return Seg{s, __ldg(ptr + s), __ldg(ptr + s + 1), -1};
 }
 
+// Chunks are handed out to warps dynamically, kWalkGrab consecutive chunks at
+// a time, from a counter in the workspace header (reset by gnn_empty_kernel):
+// a warp that meets short rows or few cut segments takes more chunks, so no
+// warp of a CTA waits long for the others.  Results do not depend on which
+// warp takes a chunk: every chunk's sums go to that chunk's slots.
+constexpr int kWalkGrab = 2;
+__device__ __forceinline__ int next_group(uint32_t* ctr, int lane) {
+  int g = 0;
+  if (lane == 0) g = (int)atomicAdd(ctr, 1u);
+  return __shfl_sync(FULL_MASK, g, 0);
+}
+
 struct ChunkPieces {
   float* __restrict__ pfirst;   // [chunks x 64]: part of a segment begun in an earlier chunk
   float* __restrict__ plast;    // [chunks x 64]: part of the segment that continues past it
@@ -255,23 +267,26 @@ __global__ void __launch_bounds__(kWideThreads, kFwdCtas)
     gnn_fwd_kernel(const int32_t* __restrict__ rowptr, const int32_t* __restrict__ colidx,
                    const float* __restrict__ val, int m, int nnz, int nchunks,
                    const float* __restrict__ P, const float* __restrict__ Z, float* __restrict__ D,
-                   float* __restrict__ dA, ChunkPieces pc, WsHeader* hdr, double* partials,
-                   double* loss_out) {
-  __shared__ double red[kWideWarps];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int gw = blockIdx.x * kWideWarps + warp, nw = gridDim.x * kWideWarps;
-  const int c0 = (int)(((long long)nchunks * gw) / nw), c1 = (int)(((long long)nchunks * (gw + 1)) / nw);
+                   float* __restrict__ dA, ChunkPieces pc, WsHeader* hdr,
+                   double* __restrict__ closs) {
+  const int lane = threadIdx.x & 31;
   FwdVisit vis{colidx, P, Z, D, WITH_DA ? dA : nullptr, pc, 0, lane, 0.0, zero4(), zero4(), -1};
-  int hint = 0;
-  for (int ch = c0; ch < c1; ++ch) {
-    const int cs = ch * kWideChunk, ce = min(cs + kWideChunk, nnz);
-    if (lane == 0) pc.lastseg[ch] = -1;
-    __syncwarp();
-    vis.ch = ch;
-    if (cs < ce) pair_walk(rowptr, m, colidx, val, P, cs, ce, hint, lane, vis, &hint);
+  const int ngroups = (nchunks + kWalkGrab - 1) / kWalkGrab;
+  while (true) {
+    const int g = next_group(&hdr->work[0], lane);
+    if (g >= ngroups) break;   // warp-uniform
+    int hint = 0;
+    for (int ch = g * kWalkGrab; ch < min((g + 1) * kWalkGrab, nchunks); ++ch) {
+      const int cs = ch * kWideChunk, ce = min(cs + kWideChunk, nnz);
+      if (lane == 0) pc.lastseg[ch] = -1;
+      __syncwarp();
+      vis.ch = ch;
+      vis.loss = 0.0;
+      if (cs < ce) pair_walk(rowptr, m, colidx, val, P, cs, ce, hint, lane, vis, &hint);
+      const double cl = warp_sum_d(vis.loss);   // this chunk's rows, added in lane order
+      if (lane == 0) closs[ch] = cl;
+    }
   }
-  const double cta = block_sum_d(vis.loss, red);
-  publish_loss(cta, hdr, partials, 0, false, 1.0, loss_out, red);
 }
 
 // ---- rows and columns without keys -----------------------------------------
@@ -287,6 +302,10 @@ __global__ void __launch_bounds__(kWideThreads)
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int half = lane >> 4, sl = lane & 15;
   const int gw = blockIdx.x * kWideWarps + warp, nw = gridDim.x * kWideWarps;
+  if (blockIdx.x == 0 && threadIdx.x == 0) {   // the walks that follow hand out chunks from 0
+    hdr->work[0] = 0;
+    hdr->work[1] = 0;
+  }
   const int nbr = (m + 31) / 32, nbc = G ? (n + 31) / 32 : 0;
   float lossf = 0.f;   // this lane's part, within 32-row blocks
   double loss = 0.0;
@@ -347,11 +366,17 @@ __global__ void __launch_bounds__(kWideThreads)
 __global__ void __launch_bounds__(kWideThreads)
     wide_fix_kernel(const int32_t* __restrict__ ptr, int nchunks, ChunkPieces pc,
                     const float* __restrict__ Z, float* __restrict__ out, WsHeader* hdr,
-                    double* partials, int first_slot, double* loss_out) {
+                    double* partials, int first_slot, const double* __restrict__ closs,
+                    double* loss_out) {
   __shared__ double red[kWideWarps];
+  __shared__ bool s_last;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int gw = blockIdx.x * kWideWarps + warp, nw = gridDim.x * kWideWarps;
   double loss = 0.0;
+  // the forward walk's per-chunk sums: this CTA adds its own slice, in order
+  if (closs)
+    for (int ch = blockIdx.x * blockDim.x + threadIdx.x; ch < nchunks; ch += gridDim.x * blockDim.x)
+      loss += closs[ch];
   for (int ch = gw; ch < nchunks; ch += nw) {
     const int s = __ldg(pc.lastseg + ch);
     if (s < 0) continue;   // warp-uniform
@@ -369,9 +394,24 @@ __global__ void __launch_bounds__(kWideThreads)
     }
     st2(out, s, lane, t);
   }
-  if (loss_out) {
-    const double cta = block_sum_d(loss, red);
-    publish_loss(cta, hdr, partials, first_slot, true, 1.0, loss_out, red);
+  if (!loss_out) return;
+  // this CTA's sum in slot first_slot + b; the last CTA adds the slots in order
+  const double cta = block_sum_d(loss, red);
+  if (threadIdx.x == 0) {
+    partials[first_slot + blockIdx.x] = cta;
+    __threadfence();
+    s_last = atomicAdd(&hdr->ticket, 1u) == gridDim.x - 1;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const volatile double* pv = partials;
+  double v = 0.0;
+  for (int i = threadIdx.x; i < first_slot + (int)gridDim.x; i += blockDim.x) v += pv[i];
+  const double tot = block_sum_d(v, red);
+  if (threadIdx.x == 0) {
+    *loss_out = tot;
+    hdr->ticket = 0;
   }
 }
 
@@ -460,10 +500,8 @@ __global__ void __launch_bounds__(kWideThreads, kColCtas)
                    const float* __restrict__ val_csc, int n, int nnz, int nchunks,
                    const float* __restrict__ D, float* __restrict__ G, ChunkPieces pc,
                    const int32_t* __restrict__ perm, const float* __restrict__ P,
-                   float* __restrict__ dA) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int gw = blockIdx.x * kWideWarps + warp, nw = gridDim.x * kWideWarps;
-  const int c0 = (int)(((long long)nchunks * gw) / nw), c1 = (int)(((long long)nchunks * (gw + 1)) / nw);
+                   float* __restrict__ dA, WsHeader* hdr) {
+  const int lane = threadIdx.x & 31;
   ColVisit vis;
   vis.G = G;
   vis.pc = pc;
@@ -479,13 +517,18 @@ __global__ void __launch_bounds__(kWideThreads, kColCtas)
   vis.pnext_c = -1;
 #pragma unroll
   for (int u = 0; u < kPairs; ++u) vis.t[u] = 0.f;
-  int hint = 0;
-  for (int ch = c0; ch < c1; ++ch) {
-    const int cs = ch * kWideChunk, ce = min(cs + kWideChunk, nnz);
-    if (lane == 0) pc.lastseg[ch] = -1;
-    __syncwarp();
-    vis.ch = ch;
-    if (cs < ce) pair_walk(colptr, n, rowidx, val_csc, D, cs, ce, hint, lane, vis, &hint);
+  const int ngroups = (nchunks + kWalkGrab - 1) / kWalkGrab;
+  while (true) {
+    const int g = next_group(&hdr->work[1], lane);
+    if (g >= ngroups) break;   // warp-uniform
+    int hint = 0;
+    for (int ch = g * kWalkGrab; ch < min((g + 1) * kWalkGrab, nchunks); ++ch) {
+      const int cs = ch * kWideChunk, ce = min(cs + kWideChunk, nnz);
+      if (lane == 0) pc.lastseg[ch] = -1;
+      __syncwarp();
+      vis.ch = ch;
+      if (cs < ce) pair_walk(colptr, n, rowidx, val_csc, D, cs, ce, hint, lane, vis, &hint);
+    }
   }
 }
 cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const float* Z,
@@ -494,10 +537,11 @@ cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const flo
   const int sms = device_sm_count();
   const int m = A->m, n = A->n, nnz = (int)A->nnz;
   const int nchunks = nnz <= 0 ? 1 : (nnz + kWideChunk - 1) / kWideChunk;
-  const int warps_per_sm = 2048 / 32;
-  // a few chunks per warp, enough warps to fill every SM
-  const int g1 = std::max(1, std::min((nchunks + kWideWarps - 1) / kWideWarps,
-                                      sms * warps_per_sm / kWideWarps * 4));
+  // the walks: as many CTAs as are resident at once (their warps take chunk
+  // groups from a counter until none is left)
+  const int ngroups = (nchunks + kWalkGrab - 1) / kWalkGrab;
+  const int gf1 = std::max(1, std::min((ngroups + kWideWarps - 1) / kWideWarps, sms * kFwdCtas));
+  const int gc1 = std::max(1, std::min((ngroups + kWideWarps - 1) / kWideWarps, sms * kColCtas));
   const int gfix = std::max(1, std::min((nchunks + kWideWarps - 1) / kWideWarps, sms * 8));
   const ChunkPieces pc{L.pfirst, L.plast, L.lastseg};
   const bool back = dH || dW || (dA && A->csc_perm);
@@ -519,15 +563,15 @@ cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const flo
   {
     KTimer t("gnn_fwd", st);
     auto fwd = (dA && !dA_in_col) ? gnn_fwd_kernel<true> : gnn_fwd_kernel<false>;
-    fwd<<<g1, kWideThreads, 0, st>>>(A->rowptr, A->colidx, A->val, m, nnz, nchunks, L.P, Z, L.D,
-                                     dA_in_col ? nullptr : dA, pc, L.hdr, L.partials + ge, loss);
+    fwd<<<gf1, kWideThreads, 0, st>>>(A->rowptr, A->colidx, A->val, m, nnz, nchunks, L.P, Z, L.D,
+                                      dA_in_col ? nullptr : dA, pc, L.hdr, L.closs);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   // 3. cut rows (also finalises the loss over every partial slot)
   {
     KTimer t("gnn_fix", st);
     wide_fix_kernel<<<gfix, kWideThreads, 0, st>>>(A->rowptr, nchunks, pc, Z, L.D, L.hdr,
-                                                   L.partials, ge + g1, loss);
+                                                   L.partials, ge, L.closs, loss);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   // 4. dA of the cut rows
@@ -541,15 +585,16 @@ cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const flo
   // 5-6. G = A^T D
   {
     KTimer t("gnn_col", st);
-    gnn_col_kernel<<<g1, kWideThreads, 0, st>>>(A->colptr, A->rowidx, A->val_csc, n, nnz,
-                                                 nchunks, L.D, L.G, pc,
-                                                 dA_in_col ? A->csc_perm : nullptr, L.P, dA);
+    gnn_col_kernel<<<gc1, kWideThreads, 0, st>>>(A->colptr, A->rowidx, A->val_csc, n, nnz,
+                                                  nchunks, L.D, L.G, pc,
+                                                  dA_in_col ? A->csc_perm : nullptr, L.P, dA,
+                                                  L.hdr);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   {
     KTimer t("gnn_col_fix", st);
     wide_fix_kernel<<<gfix, kWideThreads, 0, st>>>(A->colptr, nchunks, pc, nullptr, L.G, L.hdr,
-                                                   L.partials, 0, nullptr);
+                                                   L.partials, 0, nullptr, nullptr);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   if (!dH && !dW) return cudaSuccess;
