@@ -85,12 +85,13 @@ __device__ __forceinline__ Seg next_segment(const int32_t* __restrict__ ptr, int
   return Seg{s, __ldg(ptr + s), __ldg(ptr + s + 1), -1};
 }
 
-// Chunks are handed out to warps dynamically, kWalkGrab consecutive chunks at
-// a time, from a counter in the workspace header (reset by gnn_empty_kernel):
+// Chunks are handed out to warps dynamically, a few consecutive chunks at a
+// time, from a counter in the workspace header (reset by gnn_empty_kernel):
 // a warp that meets short rows or few cut segments takes more chunks, so no
 // warp of a CTA waits long for the others.  Results do not depend on which
 // warp takes a chunk: every chunk's sums go to that chunk's slots.
-constexpr int kWalkGrab = 2;
+constexpr int kFwdGrab = 2;   // chunks per grab, measured best for each walk
+constexpr int kColGrab = 1;
 __device__ __forceinline__ int next_group(uint32_t* ctr, int lane) {
   int g = 0;
   if (lane == 0) g = (int)atomicAdd(ctr, 1u);
@@ -271,12 +272,12 @@ __global__ void __launch_bounds__(kWideThreads, kFwdCtas)
                    double* __restrict__ closs) {
   const int lane = threadIdx.x & 31;
   FwdVisit vis{colidx, P, Z, D, WITH_DA ? dA : nullptr, pc, 0, lane, 0.0, zero4(), zero4(), -1};
-  const int ngroups = (nchunks + kWalkGrab - 1) / kWalkGrab;
+  const int ngroups = (nchunks + kFwdGrab - 1) / kFwdGrab;
   while (true) {
     const int g = next_group(&hdr->work[0], lane);
     if (g >= ngroups) break;   // warp-uniform
     int hint = 0;
-    for (int ch = g * kWalkGrab; ch < min((g + 1) * kWalkGrab, nchunks); ++ch) {
+    for (int ch = g * kFwdGrab; ch < min((g + 1) * kFwdGrab, nchunks); ++ch) {
       const int cs = ch * kWideChunk, ce = min(cs + kWideChunk, nnz);
       if (lane == 0) pc.lastseg[ch] = -1;
       __syncwarp();
@@ -517,12 +518,12 @@ __global__ void __launch_bounds__(kWideThreads, kColCtas)
   vis.pnext_c = -1;
 #pragma unroll
   for (int u = 0; u < kPairs; ++u) vis.t[u] = 0.f;
-  const int ngroups = (nchunks + kWalkGrab - 1) / kWalkGrab;
+  const int ngroups = (nchunks + kColGrab - 1) / kColGrab;
   while (true) {
     const int g = next_group(&hdr->work[1], lane);
     if (g >= ngroups) break;   // warp-uniform
     int hint = 0;
-    for (int ch = g * kWalkGrab; ch < min((g + 1) * kWalkGrab, nchunks); ++ch) {
+    for (int ch = g * kColGrab; ch < min((g + 1) * kColGrab, nchunks); ++ch) {
       const int cs = ch * kWideChunk, ce = min(cs + kWideChunk, nnz);
       if (lane == 0) pc.lastseg[ch] = -1;
       __syncwarp();
@@ -539,9 +540,10 @@ cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const flo
   const int nchunks = nnz <= 0 ? 1 : (nnz + kWideChunk - 1) / kWideChunk;
   // the walks: as many CTAs as are resident at once (their warps take chunk
   // groups from a counter until none is left)
-  const int ngroups = (nchunks + kWalkGrab - 1) / kWalkGrab;
-  const int gf1 = std::max(1, std::min((ngroups + kWideWarps - 1) / kWideWarps, sms * kFwdCtas));
-  const int gc1 = std::max(1, std::min((ngroups + kWideWarps - 1) / kWideWarps, sms * kColCtas));
+  const int fgroups = (nchunks + kFwdGrab - 1) / kFwdGrab;
+  const int cgroups = (nchunks + kColGrab - 1) / kColGrab;
+  const int gf1 = std::max(1, std::min((fgroups + kWideWarps - 1) / kWideWarps, sms * kFwdCtas));
+  const int gc1 = std::max(1, std::min((cgroups + kWideWarps - 1) / kWideWarps, sms * kColCtas));
   const int gfix = std::max(1, std::min((nchunks + kWideWarps - 1) / kWideWarps, sms * 8));
   const ChunkPieces pc{L.pfirst, L.plast, L.lastseg};
   const bool back = dH || dW || (dA && A->csc_perm);

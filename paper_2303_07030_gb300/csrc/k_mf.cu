@@ -194,6 +194,7 @@ __global__ void __launch_bounds__(256)
                     float lam, float* __restrict__ dU, float* __restrict__ dV, WsHeader* hdr,
                     double* partials) {
   __shared__ double red[8];
+  if (blockIdx.x == 0 && threadIdx.x == 0) hdr->work[0] = 0;   // the sweep's chunk counter
   const size_t nu = (size_t)m * 16, nt = nu + (size_t)n * 16;   // float4 counts
   double s = 0.0;
   for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < nt;
@@ -227,24 +228,27 @@ __global__ void __launch_bounds__(kMfaThreads)
                MfaPieces pc, WsHeader* hdr, double* partials, int first_slot) {
   __shared__ float hot[kMfHot * 64];
   __shared__ double red[kMfaWarps];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
   const int h = lane >> 4, sl = lane & 15;
   const bool ranked = rcolidx != nullptr && dV != nullptr;
   if (ranked) {
     for (int i = threadIdx.x; i < kMfHot * 64; i += blockDim.x) hot[i] = 0.f;
     __syncthreads();
   }
-  const int gw = blockIdx.x * kMfaWarps + warp, nw = gridDim.x * kMfaWarps;
-  const int c0 = (int)(((long long)nchunks * gw) / nw), c1 = (int)(((long long)nchunks * (gw + 1)) / nw);
   const int kl = batch_key_of_lane(lane);   // the key whose dot product this lane ends with
   double loss = 0.0;
-  int hint = 0;
-  for (int ch = c0; ch < c1; ++ch) {
+  // chunks are handed out one at a time from a counter in the workspace
+  // header (reset by mfa_init_kernel): hub rows make chunks very unequal
+  while (true) {
+    int ch = 0;
+    if (lane == 0) ch = (int)atomicAdd(&hdr->work[0], 1u);
+    ch = __shfl_sync(FULL_MASK, ch, 0);
+    if (ch >= nchunks) break;   // warp-uniform
     const int cs = ch * kMfaChunk, ce = min(cs + kMfaChunk, nnz);
     if (lane == 0) pc.lastseg[ch] = -1;
     __syncwarp();
     if (cs >= ce) continue;
-    int r = warp_gallop_lower_bound(rowptr, hint, m + 1, cs + 1) - 1;   // the row of key cs
+    int r = warp_lower_bound(rowptr, 0, m + 1, cs + 1) - 1;   // the row of key cs
     int s0 = __ldg(rowptr + r), s1 = __ldg(rowptr + r + 1);
     while (true) {
       const int ps = max(s0, cs), pe = min(s1, ce);
@@ -316,7 +320,6 @@ __global__ void __launch_bounds__(kMfaThreads)
       s0 = __ldg(rowptr + r);
       s1 = __ldg(rowptr + r + 1);
     }
-    hint = r;
   }
   if (ranked) {   // the hot columns' sums, once per CTA
     __syncthreads();
