@@ -426,10 +426,13 @@ sdad_status sdad_cp3_grad(const sdad_coo3* T, const float* A, const float* B, co
  *   dA_val[nnz] out, on keys(A): D_i . (H W)_j with D = Y - Z  (nullable)
  *   dH[n x f_in] out, (A^T D) W^T                              (nullable)
  *   dW[f_in x f_out] out, H^T (A^T D)                          (nullable)
- *   dH and dW need A's CSC twin (only SDAD_T_CSC / AUTO are supported).
- *   With A->csc_perm (16-byte aligned) dA is computed in the column pass over
- *   the CSC twin, which gathers D anyway (the twin is then needed for dA too);
- *   without it, in the forward pass with a second gather of (H W) rows. */
+ *   G = A^T D (for dH, dW): SDAD_T_CSC walks A's CSC twin (bit-reproducible);
+ *   SDAD_T_ATOMIC scatters it from the CSR with vector atomics (no CSC twin
+ *   needed; order not fixed); AUTO is measured (see sdad_tmode), or ATOMIC
+ *   when A has no CSC twin.
+ *   With A->csc_perm (16-byte aligned) and SDAD_T_CSC, dA is computed in the
+ *   column pass over the CSC twin, which gathers D anyway; otherwise in the
+ *   forward pass with a second gather of (H W) rows. */
 sdad_status sdad_gnn_grad(const sdad_csr* A, const float* H, const float* W, const float* Z,
                           int32_t f_in, int32_t f_out, double* loss, float* dA_val, float* dH,
                           float* dW, sdad_tmode tmode, void* ws, size_t ws_bytes, void* stream);

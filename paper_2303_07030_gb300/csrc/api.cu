@@ -660,11 +660,12 @@ sdad_status sdad_gnn_grad(const sdad_csr* A, const float* H, const float* W, con
                           int32_t f_in, int32_t f_out, double* loss, float* dA_val, float* dH,
                           float* dW, sdad_tmode tmode, void* ws, size_t ws_bytes, void* stream) {
   if (tmode < SDAD_T_AUTO || tmode > SDAD_T_ATOMIC) return SDAD_ERR_SHAPE;
-  if (tmode == SDAD_T_ATOMIC) return SDAD_ERR_UNSUPPORTED;
   if (f_in != 128 || f_out != 64) return SDAD_ERR_UNSUPPORTED;
   if (!A) return SDAD_ERR_NULL;
+  // AUTO without the CSC twin: G scattered from the CSR
+  if (tmode == SDAD_T_AUTO && (dH || dW) && !A->colptr) tmode = SDAD_T_ATOMIC;
   // the column walk runs for dH, dW, and for dA when the permutation is given
-  sdad_status s = check_csr(A, dH || dW || (dA_val && A->csc_perm));
+  sdad_status s = check_csr(A, tmode != SDAD_T_ATOMIC && (dH || dW || (dA_val && A->csc_perm)));
   if (s) return s;
   if (A->csc_perm && A->nnz > 0 && !a16(A->csc_perm)) return SDAD_ERR_ALIGN;
   if (!H || !W || !Z || !loss) return SDAD_ERR_NULL;
@@ -672,7 +673,18 @@ sdad_status sdad_gnn_grad(const sdad_csr* A, const float* H, const float* W, con
   const WsLayout L = ws_layout(SDAD_EXPR_GNN, A->m, A->n, A->nnz, f_out, ws);
   if ((s = check_ws(L, ws, ws_bytes))) return s;
   if ((s = check_device())) return s;
-  return map_cuda(run_gnn(A, H, W, Z, loss, dA_val, dH, dW, L, (cudaStream_t)stream));
+  const cudaStream_t st = (cudaStream_t)stream;
+  auto run = [&](sdad_tmode mode) {
+    return run_gnn(A, H, W, Z, loss, dA_val, dH, dW, mode == SDAD_T_ATOMIC, L, st);
+  };
+  if (tmode == SDAD_T_AUTO && (dH || dW)) {
+    const uint32_t flags = (dA_val ? 1u : 0u) | (dH ? 2u : 0u) | (dW ? 4u : 0u) |
+                           (A->csc_perm ? 8u : 0u);
+    return map_cuda(run_auto(AutoKey{0, SDAD_EXPR_GNN, A->rowptr, A->colidx, A->nnz, A->m, A->n,
+                                     flags},
+                             SDAD_T_CSC, st, run));
+  }
+  return map_cuda(run(tmode));
 }
 
 sdad_status sdad_gnn_jvp(const sdad_csr* A, const float* H, const float* W, const float* Z,

@@ -121,8 +121,8 @@ cudaError_t run_gnn_jvp(const sdad_csr* A, const float* H, const float* W, const
                         double* loss_t, const WsLayout& L, cudaStream_t st);
 
 cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const float* Z,
-                    double* loss, float* dA, float* dH, float* dW, const WsLayout& L,
-                    cudaStream_t st);
+                    double* loss, float* dA, float* dH, float* dW, bool atomic,
+                    const WsLayout& L, cudaStream_t st);
 
 // Dense projection kernels (graph loss): P = H W;  dH = G W^T and per-CTA
 // partials of H^T G;  dW = sum of the partials.

@@ -532,9 +532,46 @@ __global__ void __launch_bounds__(kWideThreads, kColCtas)
     }
   }
 }
+// ---- 5 (atomic mode): G = A^T D scattered from the CSR ----------------------
+// For each key (i, j): G_j += A_ij D_i, with the 64-wide row of D_i held by
+// the warp (lane l: elements 2l, 2l+1) while the walk is in row i, added to
+// G_j with vector atomics (float2 per lane).  Chunks of 1024 keys come from
+// the workspace's second work counter.  No CSC twin is needed; the order of
+// the additions is not fixed.
+__global__ void __launch_bounds__(kWideThreads)
+    gnn_scatter_kernel(const int32_t* __restrict__ rowptr, const int32_t* __restrict__ colidx,
+                       const float* __restrict__ val, int m, int nnz, int nchunks,
+                       const float* __restrict__ D, float* __restrict__ G, WsHeader* hdr) {
+  const int lane = threadIdx.x & 31;
+  while (true) {
+    const int ch = next_group(&hdr->work[1], lane);
+    if (ch >= nchunks) break;   // warp-uniform
+    const int cs = ch * kWideChunk, ce = min(cs + kWideChunk, nnz);
+    if (cs >= ce) continue;
+    int r = warp_lower_bound(rowptr, 0, m + 1, cs + 1) - 1;   // the row of key cs
+    int s1 = __ldg(rowptr + r + 1);
+    float2 d = ld2(D, r, lane);
+    for (int base = cs; base < ce; base += 32) {
+      const int nk = min(32, ce - base);
+      const int jl = lane < nk ? __ldg(colidx + base + lane) : 0;
+      const float al = lane < nk ? __ldg(val + base + lane) : 0.f;
+      for (int k = 0; k < nk; ++k) {
+        const int j = __shfl_sync(FULL_MASK, jl, k);
+        const float a = __shfl_sync(FULL_MASK, al, k);
+        if (base + k >= s1) {   // the key opens a later row (warp-uniform)
+          r = warp_gallop_lower_bound(rowptr, r + 1, m + 1, base + k + 1) - 1;
+          s1 = __ldg(rowptr + r + 1);
+          d = ld2(D, r, lane);
+        }
+        atomicAdd(reinterpret_cast<float2*>(G + (size_t)j * 64) + lane, make_float2(a * d.x, a * d.y));
+      }
+    }
+  }
+}
+
 cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const float* Z,
-                    double* loss, float* dA, float* dH, float* dW, const WsLayout& L,
-                    cudaStream_t st) {
+                    double* loss, float* dA, float* dH, float* dW, bool atomic,
+                    const WsLayout& L, cudaStream_t st) {
   const int sms = device_sm_count();
   const int m = A->m, n = A->n, nnz = (int)A->nnz;
   const int nchunks = nnz <= 0 ? 1 : (nnz + kWideChunk - 1) / kWideChunk;
@@ -546,10 +583,12 @@ cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const flo
   const int gc1 = std::max(1, std::min((cgroups + kWideWarps - 1) / kWideWarps, sms * kColCtas));
   const int gfix = std::max(1, std::min((nchunks + kWideWarps - 1) / kWideWarps, sms * 8));
   const ChunkPieces pc{L.pfirst, L.plast, L.lastseg};
-  const bool back = dH || dW || (dA && A->csc_perm);
+  // the column walk runs for dH and dW (and for dA when the transpose
+  // permutation is given), unless G is scattered from the CSR (atomic mode)
+  const bool back = !atomic && (dH || dW || (dA && A->csc_perm));
   // with the transpose permutation, dA comes from the column walk (which
   // gathers D anyway) instead of a second gather of P in the forward walk
-  const bool dA_in_col = dA && A->csc_perm;
+  const bool dA_in_col = !atomic && dA && A->csc_perm;
   cudaError_t e;
   // 1. P = H W
   if ((e = dense_proj_fwd(H, W, L.P, n, L.hdr, st)) != cudaSuccess) return e;
@@ -582,6 +621,18 @@ cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const flo
     gnn_cut_sddmm_kernel<<<gfix, kWideThreads, 0, st>>>(A->rowptr, A->colidx, m, nnz, nchunks,
                                                         L.P, L.D, dA);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  }
+  if (atomic) {   // 5. G = A^T D scattered from the CSR
+    if (!dH && !dW) return cudaSuccess;
+    if ((e = zero_f32(L.G, (size_t)n * 64, st)) != cudaSuccess) return e;
+    if (nnz > 0) {
+      const int gs = std::max(1, std::min((nchunks + kWideWarps - 1) / kWideWarps, sms * 8));
+      KTimer t("gnn_scatter", st);
+      gnn_scatter_kernel<<<gs, kWideThreads, 0, st>>>(A->rowptr, A->colidx, A->val, m, nnz,
+                                                       nchunks, L.D, L.G, L.hdr);
+      if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    return dense_proj_bwd(H, W, L.G, dH, L.dWpart, dW, n, L.hdr, st);
   }
   if (!back) return cudaSuccess;
   // 5-6. G = A^T D

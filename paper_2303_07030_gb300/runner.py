@@ -206,8 +206,10 @@ class Cp3Run(_Base):
 class GnnRun(_Base):
     expr = S.SDAD_EXPR_GNN
 
-    def __init__(self, p, want_dA=True, with_perm=True, device="cuda"):
-        self.p, self.device = p, device
+    def __init__(self, p, want_dA=True, with_perm=True, tmode=S.SDAD_T_AUTO, device="cuda"):
+        """tmode: SDAD_T_CSC (G = A^T D by the column walk over the CSC twin),
+        SDAD_T_ATOMIC (G scattered from the CSR) or AUTO (measured)."""
+        self.p, self.device, self.tmode = p, device, tmode
         self.f_in, self.f_out = int(p.params["f_in"]), int(p.params["f_out"])
         self.A = S.CsrDevice(p.m, p.n, p.row, p.col, p.val, csc=True, with_perm=with_perm,
                              device=device)

@@ -94,3 +94,14 @@ def test_default_headline_is_the_largest_workload():
         sys.argv = sys_argv
     assert a.config == "gnn" and a.others == "all"
     assert set(bench.ALL_CONFIGS) == set(bench.WORKLOAD_NAMES)
+
+
+def test_sweep_covers_density_and_dimension():
+    kinds = {(cfg, what) for cfg, _, what in bench.SWEEP}
+    assert ("lsq", "density") in kinds and ("lsq", "dimension") in kinds
+    assert ("logreg", "density") in kinds and ("gnn", "dimension") in kinds
+    # every point is a valid generator call of its workload (sizes only checked here)
+    for cfg, ov, _ in bench.SWEEP:
+        assert cfg in bench.WORKLOAD_NAMES and isinstance(ov, dict) and ov
+    d = [ov["draws"] for cfg, ov, w in bench.SWEEP if cfg == "lsq" and w == "density"]
+    assert d == sorted(d) and len(set(d)) == len(d)

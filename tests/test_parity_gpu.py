@@ -119,12 +119,28 @@ def test_cp3_small(tmode):
     assert_close(out, oracle_for("cp3", p), ["dA", "dB", "dC", "dT"])
 
 
-@pytest.mark.parametrize("with_perm", [True, False])   # dA in the column walk, or the forward walk
-def test_gnn_small(with_perm):
+# dA in the column walk (transpose permutation) or in the forward walk; G by
+# the column walk, scattered from the CSR (atomic), or as AUTO measures
+@pytest.mark.parametrize("kw", [{"with_perm": True, "tmode": S.SDAD_T_CSC},
+                                {"with_perm": False, "tmode": S.SDAD_T_CSC},
+                                {"with_perm": True, "tmode": S.SDAD_T_ATOMIC},
+                                {"with_perm": True, "tmode": S.SDAD_T_AUTO}])
+def test_gnn_small(kw):
     p = W.make("gnn", "small")
-    r, out = run("gnn", p, with_perm=with_perm)
+    r, out = run("gnn", p, **kw)
     pattern_matches(r, p)
     assert_close(out, oracle_for("gnn", p), COMPARED["gnn"])
+
+
+def test_gnn_without_csc_twin():
+    # AUTO on a graph without its CSC twin scatters G from the CSR
+    p = W.make("gnn", "small")
+    r = R.GnnRun(p, with_perm=False)
+    r.desc.colptr = r.desc.rowidx = r.desc.val_csc = None
+    r.step()
+    torch.cuda.synchronize()
+    r.check()
+    assert_close(r.outputs(), oracle_for("gnn", p), COMPARED["gnn"])
 
 
 # ----------------------------------------------------------------------------
@@ -221,8 +237,9 @@ def test_cp3_hub_index():
         assert_close(out, oracle_for("cp3", p), ["dA", "dB", "dC", "dT"])
 
 
-@pytest.mark.parametrize("with_perm", [True, False])
-def test_gnn_hub_rows_columns_and_empty_rows(with_perm):
+@pytest.mark.parametrize("kw", [{"with_perm": True}, {"with_perm": False},
+                                {"with_perm": True, "tmode": S.SDAD_T_ATOMIC}])
+def test_gnn_hub_rows_columns_and_empty_rows(kw):
     # row 0 holds 3000 keys (> one chunk), column 5 holds every even row
     # (a long column part), rows in the upper half with odd index are empty
     rng = np.random.default_rng(6)
@@ -238,7 +255,7 @@ def test_gnn_hub_rows_columns_and_empty_rows(with_perm):
                 "Z": rng.standard_normal((nv, 64)).astype(np.float32)},
                {"f_in": 128, "f_out": 64})
     assert (np.bincount(row, minlength=nv) == 0).any()
-    _, out = run("gnn", p, with_perm=with_perm)
+    _, out = run("gnn", p, **kw)
     assert_close(out, oracle_for("gnn", p), COMPARED["gnn"])
 
 
