@@ -47,8 +47,17 @@ constexpr bool kWalkLookahead = SDAD_WALK_LOOKAHEAD;
 // Resident CTAs per SM the walks are compiled for: the forward walk measured
 // fastest at 4 (64 registers), the column walk (which also holds P_c and the
 // batch's dot products) at 3.
-constexpr int kFwdCtas = 4;
+#ifndef SDAD_FWD_CTAS
+#define SDAD_FWD_CTAS 4
+#endif
+#ifndef SDAD_FWD_PAIRS
+#define SDAD_FWD_PAIRS 8
+#endif
+constexpr int kFwdCtas = SDAD_FWD_CTAS;
 constexpr int kColCtas = 3;
+// key pairs gathered per batch by the forward walk (the column walk reduces
+// its dot products in batches of kPairs)
+constexpr int kFwdPairs = SDAD_FWD_PAIRS;
 
 __device__ __forceinline__ float2 ld2(const float* base, int r, int lane) {
   return __ldg(reinterpret_cast<const float2*>(base + (size_t)r * 64) + lane);
@@ -126,7 +135,7 @@ struct ChunkPieces {
 // vis.key(h, x, q) for every key q (x = the gathered row, held by half h) at
 // the moment the walk is in q's segment.  Segments without keys are skipped
 // (gnn_empty_kernel handles them).
-template <class Vis>
+template <int NP, class Vis>
 __device__ __forceinline__ void pair_walk(const int32_t* __restrict__ ptr, int nseg,
                                           const int32_t* __restrict__ idx,
                                           const float* __restrict__ val,
@@ -143,16 +152,16 @@ __device__ __forceinline__ void pair_walk(const int32_t* __restrict__ ptr, int n
     const int jl = lane < nk ? __ldg(idx + base + lane) : 0;
     const float al = lane < nk ? __ldg(val + base + lane) : 0.f;
     vis.window(base, nk, lane);
-    for (int k0 = 0; k0 < nk; k0 += 2 * kPairs) {
-      float4 x[kPairs];
+    for (int k0 = 0; k0 < nk; k0 += 2 * NP) {
+      float4 x[NP];
 #pragma unroll
-      for (int u = 0; u < kPairs; ++u) {
+      for (int u = 0; u < NP; ++u) {
         const int kk = k0 + 2 * u + h;
         const int j = __shfl_sync(FULL_MASK, jl, kk & 31);
         x[u] = kk < nk ? ld4(X, j, sl) : zero4();
       }
 #pragma unroll
-      for (int u = 0; u < kPairs; ++u) {
+      for (int u = 0; u < NP; ++u) {
         const int kk = k0 + 2 * u;   // this pair: keys kk (half 0) and kk + 1 (half 1)
         const float a = __shfl_sync(FULL_MASK, al, (kk + h) & 31);
         if (kk >= nk) break;   // warp-uniform
@@ -283,7 +292,7 @@ __global__ void __launch_bounds__(kWideThreads, kFwdCtas)
       __syncwarp();
       vis.ch = ch;
       vis.loss = 0.0;
-      if (cs < ce) pair_walk(rowptr, m, colidx, val, P, cs, ce, hint, lane, vis, &hint);
+      if (cs < ce) pair_walk<kFwdPairs>(rowptr, m, colidx, val, P, cs, ce, hint, lane, vis, &hint);
       const double cl = warp_sum_d(vis.loss);   // this chunk's rows, added in lane order
       if (lane == 0) closs[ch] = cl;
     }
@@ -528,7 +537,7 @@ __global__ void __launch_bounds__(kWideThreads, kColCtas)
       if (lane == 0) pc.lastseg[ch] = -1;
       __syncwarp();
       vis.ch = ch;
-      if (cs < ce) pair_walk(colptr, n, rowidx, val_csc, D, cs, ce, hint, lane, vis, &hint);
+      if (cs < ce) pair_walk<kPairs>(colptr, n, rowidx, val_csc, D, cs, ce, hint, lane, vis, &hint);
     }
   }
 }
