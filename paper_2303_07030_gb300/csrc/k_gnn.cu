@@ -44,14 +44,15 @@ constexpr int kWideWarps = kWideThreads / 32;
 #define SDAD_WALK_LOOKAHEAD 0
 #endif
 constexpr bool kWalkLookahead = SDAD_WALK_LOOKAHEAD;
-// Resident CTAs per SM the walks are compiled for: the forward walk measured
-// fastest at 4 (64 registers), the column walk (which also holds P_c and the
-// batch's dot products) at 3.
+// Resident CTAs per SM the walks are compiled for, and the forward walk's
+// batch: measured fastest with 4 key pairs per batch at 6 CTAs (40
+// registers) for the forward walk, and 8 pairs at 3 CTAs for the column walk
+// (which also holds P_c and the batch's dot products).
 #ifndef SDAD_FWD_CTAS
-#define SDAD_FWD_CTAS 4
+#define SDAD_FWD_CTAS 6
 #endif
 #ifndef SDAD_FWD_PAIRS
-#define SDAD_FWD_PAIRS 8
+#define SDAD_FWD_PAIRS 4
 #endif
 constexpr int kFwdCtas = SDAD_FWD_CTAS;
 constexpr int kColCtas = 3;
