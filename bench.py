@@ -228,6 +228,11 @@ def measured_traffic(cfg, kernel, nnz, layout=None):
                 return None, None
     except OSError:
         return None, None
+    if "bytes_per_launch" in ent:   # captured on the full workload itself
+        if ent.get("nnz") != nnz:
+            return None, None
+        b = ent["bytes_per_launch"].get(kernel)
+        return (None, None) if b is None else (int(b), ent["capture"])
     b = ent["bytes_per_key"].get(kernel)
     return (None, None) if b is None else (int(round(b * nnz)), ent["capture"])
 

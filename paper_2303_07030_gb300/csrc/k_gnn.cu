@@ -40,6 +40,23 @@ constexpr int kWideWarps = kWideThreads / 32;
 // Loading the next row's Z (forward walk) or the next column's P row (column
 // walk) one segment ahead measured neutral to slightly slower on the R-MAT
 // graph (registers); kept as an option.
+// Streamed arrays of the walks (key indices, values, permutation, Z; dA and
+// G written) read and written with the evict-first cache hint, so that L2
+// keeps more of the gathered P and D rows.
+#ifndef SDAD_WALK_STREAM_HINTS
+#define SDAD_WALK_STREAM_HINTS 0
+#endif
+constexpr bool kStreamHints = SDAD_WALK_STREAM_HINTS;
+template <class T>
+__device__ __forceinline__ T ld_stream(const T* p) {
+  return kStreamHints ? __ldcs(p) : __ldg(p);
+}
+template <class T>
+__device__ __forceinline__ void st_stream(T* p, T v) {
+  if (kStreamHints) __stcs(p, v);
+  else *p = v;
+}
+
 #ifndef SDAD_WALK_LOOKAHEAD
 #define SDAD_WALK_LOOKAHEAD 0
 #endif
@@ -150,8 +167,8 @@ __device__ __forceinline__ void pair_walk(const int32_t* __restrict__ ptr, int n
   float4 acc = zero4();
   for (int base = cs; base < ce; base += 32) {
     const int nk = min(32, ce - base);
-    const int jl = lane < nk ? __ldg(idx + base + lane) : 0;
-    const float al = lane < nk ? __ldg(val + base + lane) : 0.f;
+    const int jl = lane < nk ? ld_stream(idx + base + lane) : 0;
+    const float al = lane < nk ? ld_stream(val + base + lane) : 0.f;
     vis.window(base, nk, lane);
     for (int k0 = 0; k0 < nk; k0 += 2 * NP) {
       float4 x[NP];
@@ -249,7 +266,7 @@ struct FwdVisit {
   __device__ __forceinline__ void begin(int r, int after) {
     if (!kWalkLookahead) return;   // Z is then read when the row ends
     const int sl = lane & 15;
-    zr = r == znext_r ? znext : ld4(Z, r, sl);
+    zr = r == znext_r ? znext : ld_stream(reinterpret_cast<const float4*>(Z + (size_t)r * 64) + sl);
     znext_r = after;
     if (after >= 0) znext = ld4(Z, after, sl);
   }
@@ -260,7 +277,7 @@ struct FwdVisit {
   __device__ __forceinline__ void segment(int r, int s0, int s1, float4 tot, int cs, int ce) {
     if (pc.cut(ch, r, s0, s1, cs, ce, tot, lane)) return;
     const int sl = lane & 15;
-    if (!kWalkLookahead) zr = ld4(Z, r, sl);
+    if (!kWalkLookahead) zr = ld_stream(reinterpret_cast<const float4*>(Z + (size_t)r * 64) + sl);
     const float4 d = make_float4(tot.x - zr.x, tot.y - zr.y, tot.z - zr.z, tot.w - zr.w);
     if (lane < 16) {
       st4(D, r, sl, d);
@@ -480,7 +497,7 @@ struct ColVisit {
     if (after >= 0) pnext = ld4(P, after, sl);
   }
   __device__ __forceinline__ void window(int base, int nk, int lane_) {
-    if (perm) ql = lane_ < nk ? __ldg(perm + base + lane_) : 0;
+    if (perm) ql = lane_ < nk ? ld_stream(perm + base + lane_) : 0;
   }
   __device__ __forceinline__ void key(int, float4 x, int, int u) {
     if (perm) t[u] = dot4(x, pcol);
@@ -495,13 +512,13 @@ struct ColVisit {
     const int sl = lane_ & 15;
     const int kk = k0 + 2 * ((sl >> 1) & 7) + (lane_ >> 4);
     const int q = __shfl_sync(FULL_MASK, ql, kk & 31);
-    if ((sl & 1) == 0 && kk < nk) dA[q] = r;
+    if ((sl & 1) == 0 && kk < nk) st_stream(dA + q, r);
 #pragma unroll
     for (int u = 0; u < kPairs; ++u) t[u] = 0.f;
   }
   __device__ __forceinline__ void segment(int c, int s0, int s1, float4 tot, int cs, int ce) {
     if (pc.cut(ch, c, s0, s1, cs, ce, tot, lane)) return;
-    if (lane < 16) st4(G, c, lane, tot);
+    if (lane < 16) st_stream(reinterpret_cast<float4*>(G + (size_t)c * 64) + lane, tot);
   }
 };
 
