@@ -44,7 +44,7 @@ constexpr int kWideWarps = kWideThreads / 32;
 // G written) read and written with the evict-first cache hint, so that L2
 // keeps more of the gathered P and D rows.
 #ifndef SDAD_WALK_STREAM_HINTS
-#define SDAD_WALK_STREAM_HINTS 0
+#define SDAD_WALK_STREAM_HINTS 1
 #endif
 constexpr bool kStreamHints = SDAD_WALK_STREAM_HINTS;
 template <class T>

@@ -106,3 +106,19 @@ def test_ranked_csc_is_bit_reproducible_and_atomic_loss_is_stable():
         losses.append(q.outputs()["loss"])
     q.check()
     assert losses[1] == losses[0] and losses[2] == losses[0]
+
+
+# A larger instance (70,000 rows, 60,000 Zipf columns), in every mode, with
+# dX (the emitting variant of the row pass) and without.
+@pytest.mark.parametrize("tmode", MODES)
+@pytest.mark.parametrize("want_dX", [False, True])
+def test_logreg_ranked_larger(tmode, want_dX):
+    p = W.make("logreg", "small", m=70000, n=60000, mean_row=20.0)
+    _, out = run("logreg", p, tmode=tmode, want_dX=want_dX)
+    assert_close(out, oracle_for("logreg", p), ["dw", "dX"] if want_dX else ["dw"])
+
+
+def test_lsq_ranked_larger():
+    p = W.lsq_problem(m=70000, n=50000, draws=800000, seed=99)
+    _, out = run("lsq", p, tmode=S.SDAD_T_CSC)
+    assert_close(out, oracle_for("lsq", p), COMPARED["lsq"])
