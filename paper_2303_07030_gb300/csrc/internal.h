@@ -38,6 +38,7 @@ struct WsLayout {
   float* G;           // graph: A^T D                              [cols x f_out]
   float* dWpart;      // graph: per-CTA partial H^T G              [kDwParts x f_in x f_out]
   double* closs;      // graph: loss terms of the rows finished inside each chunk [chunks]
+  int32_t* order;     // graph: the walks' chunk-group order, then its scratch    [4 x chunks]
   float* tfirst;      // graph, forward mode: pieces of Y' (as pfirst / plast below)
   float* tlast;
   // pieces of segments cut by chunk boundaries (deterministic combination):

@@ -124,6 +124,106 @@ __device__ __forceinline__ int next_group(uint32_t* ctr, int lane) {
   if (lane == 0) g = (int)atomicAdd(ctr, 1u);
   return __shfl_sync(FULL_MASK, g, 0);
 }
+// Order of the chunk groups.  A group's walk time grows with the segments it
+// meets, not only with its keys: each segment end is a chain of dependent
+// loads (the next pointers, the Z row or the P row), while the keys of one
+// long segment stream.  On a graph whose light rows lie together (R-MAT
+// without a vertex permutation puts them at the high numbers) the groups
+// handed out last were the slowest, and a few warps ran on long after the
+// others.  So the groups that meet at least four times the mean number of
+// segments are handed out first, the others after them; both keep their
+// matrix order, so the warps in flight still work on neighbouring groups,
+// which share more of their gathered rows in L2 (sorting all groups by
+// their segment count made the column walk a seventh slower).  The order
+// changes no result: every chunk writes its own slots, which the fix kernels
+// add in chunk order.
+constexpr int kOrderThreads = 1024;
+
+struct GroupWalk {   // one walk's groups, for the order kernels
+  const int32_t* ptr;   // segment pointers (rowptr or colptr)
+  int nseg, keys, ngroups;
+  int thr;              // segments that make a group heavy
+  int32_t* order;       // [ngroups]
+};
+
+// CTA b orders groups [1024 b', 1024 b' + 1024) of walk 0 (b' = b) or of walk
+// 1 (b' = b - ctas0).  flag[g]: the group is heavy; count[b]: heavy groups of
+// the CTA.
+__global__ void __launch_bounds__(kOrderThreads)
+    group_flag_kernel(GroupWalk w0, GroupWalk w1, int ctas0, int nnz, int8_t* __restrict__ flag,
+                      int32_t* __restrict__ count) {
+  const bool second = (int)blockIdx.x >= ctas0;
+  const GroupWalk& w = second ? w1 : w0;
+  const int g = ((int)blockIdx.x - (second ? ctas0 : 0)) * kOrderThreads + threadIdx.x;
+  bool heavy = false;
+  if (g < w.ngroups) {
+    const long long cs = (long long)g * w.keys, ce = std::min<long long>(cs + w.keys, nnz);
+    if (cs < ce) {
+      // the last s with ptr[s] <= x, for x = cs and x = ce - 1
+      auto seg_of = [&](long long x) {
+        int lo = 0, hi = w.nseg + 1;   // ptr[lo] <= x < ptr[hi] (ptr[nseg + 1] taken as +inf)
+        while (hi - lo > 1) {
+          const int mid = (lo + hi) >> 1;
+          if (__ldg(w.ptr + mid) <= x) lo = mid;
+          else hi = mid;
+        }
+        return lo;
+      };
+      heavy = seg_of(ce - 1) - seg_of(cs) + 1 >= w.thr;
+    }
+    flag[(second ? w0.ngroups : 0) + g] = heavy;
+  }
+  const int c = __syncthreads_count(heavy);
+  if (threadIdx.x == 0) count[blockIdx.x] = c;
+}
+
+// Places each group: the heavy ones first, then the others, each in matrix order.
+__global__ void __launch_bounds__(kOrderThreads)
+    group_place_kernel(GroupWalk w0, GroupWalk w1, int ctas0, int ctas1,
+                       const int8_t* __restrict__ flag, const int32_t* __restrict__ count) {
+  __shared__ int part[kOrderThreads / 32][2];
+  __shared__ int tot[2];
+  const bool second = (int)blockIdx.x >= ctas0;
+  const GroupWalk& w = second ? w1 : w0;
+  const int b = (int)blockIdx.x - (second ? ctas0 : 0);
+  const int32_t* cnt = count + (second ? ctas0 : 0);
+  const int nb = second ? ctas1 : ctas0;
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  // heavy groups of the walk before this CTA's, and in all
+  int before = 0, all = 0;
+  for (int i = t; i < nb; i += kOrderThreads) {
+    const int v = __ldg(cnt + i);
+    all += v;
+    if (i < b) before += v;
+  }
+#pragma unroll
+  for (int o = 16; o; o >>= 1) {
+    before += __shfl_xor_sync(FULL_MASK, before, o);
+    all += __shfl_xor_sync(FULL_MASK, all, o);
+  }
+  if (lane == 0) { part[warp][0] = before; part[warp][1] = all; }
+  __syncthreads();
+  if (t < 2) {
+    int x = 0;
+    for (int i = 0; i < kOrderThreads / 32; ++i) x += part[i][t];
+    tot[t] = x;
+  }
+  __syncthreads();
+  const int hbefore = tot[0], hall = tot[1];
+  const int g = b * kOrderThreads + t;
+  const bool heavy = g < w.ngroups && flag[(second ? w0.ngroups : 0) + g];
+  // rank of this group among the CTA's heavy groups
+  const unsigned bal = __ballot_sync(FULL_MASK, heavy);
+  __syncthreads();
+  if (lane == 0) part[warp][0] = __popc(bal);
+  __syncthreads();
+  int rank = __popc(bal & ((1u << lane) - 1));
+  for (int i = 0; i < warp; ++i) rank += part[i][0];
+  if (g < w.ngroups) {
+    const int hrank = hbefore + rank;                        // heavy groups before g
+    w.order[heavy ? hrank : hall + (g - hrank)] = g;
+  }
+}
 
 struct ChunkPieces {
   float* __restrict__ pfirst;   // [chunks x 64]: part of a segment begun in an earlier chunk
@@ -296,13 +396,15 @@ __global__ void __launch_bounds__(kWideThreads, kFwdCtas)
                    const float* __restrict__ val, int m, int nnz, int nchunks,
                    const float* __restrict__ P, const float* __restrict__ Z, float* __restrict__ D,
                    float* __restrict__ dA, ChunkPieces pc, WsHeader* hdr,
-                   double* __restrict__ closs) {
+                   double* __restrict__ closs,
+                   const int32_t* __restrict__ order) {
   const int lane = threadIdx.x & 31;
   FwdVisit vis{colidx, P, Z, D, WITH_DA ? dA : nullptr, pc, 0, lane, 0.0, zero4(), zero4(), -1};
   const int ngroups = (nchunks + kFwdGrab - 1) / kFwdGrab;
   while (true) {
-    const int g = next_group(&hdr->work[0], lane);
-    if (g >= ngroups) break;   // warp-uniform
+    const int k = next_group(&hdr->work[0], lane);
+    if (k >= ngroups) break;   // warp-uniform
+    const int g = __ldg(order + k);
     int hint = 0;
     for (int ch = g * kFwdGrab; ch < min((g + 1) * kFwdGrab, nchunks); ++ch) {
       const int cs = ch * kWideChunk, ce = min(cs + kWideChunk, nnz);
@@ -528,7 +630,8 @@ __global__ void __launch_bounds__(kWideThreads, kColCtas)
                    const float* __restrict__ val_csc, int n, int nnz, int nchunks,
                    const float* __restrict__ D, float* __restrict__ G, ChunkPieces pc,
                    const int32_t* __restrict__ perm, const float* __restrict__ P,
-                   float* __restrict__ dA, WsHeader* hdr) {
+                   float* __restrict__ dA, WsHeader* hdr,
+                   const int32_t* __restrict__ order) {
   const int lane = threadIdx.x & 31;
   ColVisit vis;
   vis.G = G;
@@ -547,8 +650,9 @@ __global__ void __launch_bounds__(kWideThreads, kColCtas)
   for (int u = 0; u < kPairs; ++u) vis.t[u] = 0.f;
   const int ngroups = (nchunks + kColGrab - 1) / kColGrab;
   while (true) {
-    const int g = next_group(&hdr->work[1], lane);
-    if (g >= ngroups) break;   // warp-uniform
+    const int k = next_group(&hdr->work[1], lane);
+    if (k >= ngroups) break;   // warp-uniform
+    const int g = __ldg(order + k);
     int hint = 0;
     for (int ch = g * kColGrab; ch < min((g + 1) * kColGrab, nchunks); ++ch) {
       const int cs = ch * kWideChunk, ce = min(cs + kWideChunk, nnz);
@@ -619,6 +723,26 @@ cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const flo
   cudaError_t e;
   // 1. P = H W
   if ((e = dense_proj_fwd(H, W, L.P, n, L.hdr, st)) != cudaSuccess) return e;
+  // the walks' group order
+  {
+    KTimer t("gnn_order", st);
+    const int cg = back ? cgroups : 0;
+    // mean segments per group: about (segments + groups) / groups
+    const GroupWalk w0{A->rowptr, m, kFwdGrab * kWideChunk, fgroups,
+                       (int)std::min<long long>(INT_MAX, 4 * (((long long)m + fgroups + fgroups - 1) / fgroups)),
+                       L.order};
+    const GroupWalk w1{A->colptr, n, kColGrab * kWideChunk, cg,
+                       (int)std::min<long long>(INT_MAX, 4 * (((long long)n + cg + std::max(cg, 1) - 1) / std::max(cg, 1))),
+                       L.order + fgroups};
+    const int ctas0 = (fgroups + kOrderThreads - 1) / kOrderThreads;
+    const int ctas1 = (cg + kOrderThreads - 1) / kOrderThreads;
+    int8_t* flag = reinterpret_cast<int8_t*>(L.order + fgroups + cg);
+    int32_t* count = L.order + fgroups + cg + (fgroups + cg + 3) / 4;
+    group_flag_kernel<<<ctas0 + ctas1, kOrderThreads, 0, st>>>(w0, w1, ctas0, nnz, flag, count);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    group_place_kernel<<<ctas0 + ctas1, kOrderThreads, 0, st>>>(w0, w1, ctas0, ctas1, flag, count);
+  }
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
   // 2a. rows (and columns) without keys
   const int ge = std::max(1, std::min((m + n + 255) / 256, sms * 8));
   {
@@ -632,7 +756,7 @@ cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const flo
     KTimer t("gnn_fwd", st);
     auto fwd = (dA && !dA_in_col) ? gnn_fwd_kernel<true> : gnn_fwd_kernel<false>;
     fwd<<<gf1, kWideThreads, 0, st>>>(A->rowptr, A->colidx, A->val, m, nnz, nchunks, L.P, Z, L.D,
-                                      dA_in_col ? nullptr : dA, pc, L.hdr, L.closs);
+                                      dA_in_col ? nullptr : dA, pc, L.hdr, L.closs, L.order);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   // 3. cut rows (also finalises the loss over every partial slot)
@@ -668,7 +792,7 @@ cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const flo
     gnn_col_kernel<<<gc1, kWideThreads, 0, st>>>(A->colptr, A->rowidx, A->val_csc, n, nnz,
                                                   nchunks, L.D, L.G, pc,
                                                   dA_in_col ? A->csc_perm : nullptr, L.P, dA,
-                                                  L.hdr);
+                                                  L.hdr, L.order + fgroups);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   {
