@@ -2,8 +2,8 @@
 //
 // Kernel sequence of one call:
 //   1. P = H W                                           (dense projection)
-//   2. rows without keys: D_r = -Z_r and their loss term (columns without
-//      keys: G_c = 0), then the forward walk over the CSR (one warp per
+//   2. rows without keys: their loss term |Z_r|^2 / 2 (columns without
+//      keys: G_c = 0), then, in the walks' group order, the forward walk over the CSR (one warp per
 //      1024-key chunk): Y_r = sum_p val[p] P[colidx[p]];  rows finished inside
 //      the chunk: D_r = Y_r - Z_r, loss += |D_r|^2 / 2, dA[p] = D_r . P[colidx[p]];
 //      rows cut by chunk boundaries: one 64-wide piece per chunk
@@ -61,6 +61,33 @@ __device__ __forceinline__ void st_stream(T* p, T v) {
 #define SDAD_WALK_LOOKAHEAD 0
 #endif
 constexpr bool kWalkLookahead = SDAD_WALK_LOOKAHEAD;
+// Prefetch into L2 the row each upcoming segment reads when it ends (forward
+// walk: Z) or begins (column walk: P), for the segments of each window of 32
+// pointers the segment search loads.  Measured: forward walk 1.84 -> 1.70 ms
+// on the 2^22-vertex R-MAT graph (0.74 -> 0.60 ms on 2^16 vertices, where one
+// chunk of light rows sets the time); column walk 2.81 -> 3.00 ms, so off there.
+#ifndef SDAD_FWD_PREFETCH
+#define SDAD_FWD_PREFETCH 1
+#endif
+#ifndef SDAD_COL_PREFETCH
+#define SDAD_COL_PREFETCH 0
+#endif
+__device__ __forceinline__ void prefetch_l2(const void* p) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+// lane l of a window of pointers ptr[lo + 1 + l] = pv: prefetches the 256-byte
+// row of segment lo + l (l > 0) of X when that segment holds keys and lies past
+// *front; then moves *front to the window's end
+__device__ __forceinline__ void prefetch_window(const float* X, int lo, int pv, int lane, int* front) {
+  const int prev = __shfl_up_sync(FULL_MASK, pv, 1);
+  const int r = lo + lane;
+  if (lane > 0 && r > *front && pv != INT_MAX && prev < pv) {
+    const char* a = reinterpret_cast<const char*>(X + (size_t)r * 64);
+    prefetch_l2(a);
+    prefetch_l2(a + 128);
+  }
+  *front = max(*front, lo + 31);
+}
 // Resident CTAs per SM the walks are compiled for, and the forward walk's
 // batch: measured fastest with 4 key pairs per batch at 6 CTAs (40
 // registers) for the forward walk, and 8 pairs at 3 CTAs for the column walk
@@ -72,7 +99,10 @@ constexpr bool kWalkLookahead = SDAD_WALK_LOOKAHEAD;
 #define SDAD_FWD_PAIRS 4
 #endif
 constexpr int kFwdCtas = SDAD_FWD_CTAS;
-constexpr int kColCtas = 3;
+#ifndef SDAD_COL_CTAS
+#define SDAD_COL_CTAS 3
+#endif
+constexpr int kColCtas = SDAD_COL_CTAS;
 // key pairs gathered per batch by the forward walk (the column walk reduces
 // its dot products in batches of kPairs)
 constexpr int kFwdPairs = SDAD_FWD_PAIRS;
@@ -92,11 +122,13 @@ struct Seg {
   int s, s0, s1;
   int after;   // the segment after s that holds keys, when it lies in the same 32 pointers; else -1
 };
+template <class Vis>
 __device__ __forceinline__ Seg next_segment(const int32_t* __restrict__ ptr, int nseg, int lo,
-                                            int p, int lane) {
+                                            int p, int lane, Vis& vis) {
   // first i in [lo + 1, nseg] with ptr[i] > p; the segment is i - 1
   const int i = lo + 1 + lane;
   const int pv = i <= nseg ? __ldg(ptr + i) : INT_MAX;
+  vis.ahead(lo, pv, lane);
   const unsigned b = __ballot_sync(FULL_MASK, pv > p);
   if (b) {
     const int f = __ffs(b) - 1;
@@ -118,7 +150,10 @@ __device__ __forceinline__ Seg next_segment(const int32_t* __restrict__ ptr, int
 // warp of a CTA waits long for the others.  Results do not depend on which
 // warp takes a chunk: every chunk's sums go to that chunk's slots.
 constexpr int kFwdGrab = 2;   // chunks per grab, measured best for each walk
-constexpr int kColGrab = 1;
+#ifndef SDAD_COL_GRAB
+#define SDAD_COL_GRAB 1
+#endif
+constexpr int kColGrab = SDAD_COL_GRAB;
 __device__ __forceinline__ int next_group(uint32_t* ctr, int lane) {
   int g = 0;
   if (lane == 0) g = (int)atomicAdd(ctr, 1u);
@@ -138,6 +173,10 @@ __device__ __forceinline__ int next_group(uint32_t* ctr, int lane) {
 // changes no result: every chunk writes its own slots, which the fix kernels
 // add in chunk order.
 constexpr int kOrderThreads = 1024;
+#ifndef SDAD_ORDER_HEAVY
+#define SDAD_ORDER_HEAVY 4
+#endif
+constexpr int kOrderHeavy = SDAD_ORDER_HEAVY;   // heavy: at least this many times the mean
 
 struct GroupWalk {   // one walk's groups, for the order kernels
   const int32_t* ptr;   // segment pointers (rowptr or colptr)
@@ -263,6 +302,7 @@ __device__ __forceinline__ void pair_walk(const int32_t* __restrict__ ptr, int n
   // the segment holding key cs: the last s with ptr[s] <= cs
   int s = warp_gallop_lower_bound(ptr, hint, nseg + 1, cs + 1) - 1;
   int s0 = __ldg(ptr + s), s1 = __ldg(ptr + s + 1);
+  vis.front = s;
   vis.begin(s, -1);
   float4 acc = zero4();
   for (int base = cs; base < ce; base += 32) {
@@ -293,7 +333,7 @@ __device__ __forceinline__ void pair_walk(const int32_t* __restrict__ ptr, int n
         // a segment ends inside the pair
         if (p0 >= s1) {
           vis.segment(s, s0, s1, join_halves(acc), cs, ce);
-          const Seg g = next_segment(ptr, nseg, s, p0, lane);
+          const Seg g = next_segment(ptr, nseg, s, p0, lane, vis);
           s = g.s; s0 = g.s0; s1 = g.s1;
           vis.begin(s, g.after);
           acc = zero4();
@@ -303,7 +343,7 @@ __device__ __forceinline__ void pair_walk(const int32_t* __restrict__ ptr, int n
         if (two) {
           if (p0 + 1 >= s1) {
             vis.segment(s, s0, s1, join_halves(acc), cs, ce);
-            const Seg g = next_segment(ptr, nseg, s, p0 + 1, lane);
+            const Seg g = next_segment(ptr, nseg, s, p0 + 1, lane, vis);
             s = g.s; s0 = g.s0; s1 = g.s1;
             vis.begin(s, g.after);
             acc = zero4();
@@ -362,6 +402,11 @@ struct FwdVisit {
   float4 zr;     // Z row of the open row (loaded when the row begins)
   float4 znext;  // Z row of row znext_r, loaded one row ahead
   int znext_r;
+  int front;     // rows up to this one are prefetched
+
+  __device__ __forceinline__ void ahead(int lo, int pv, int lane_) {
+    if (SDAD_FWD_PREFETCH) prefetch_window(Z, lo, pv, lane_, &front);
+  }
 
   __device__ __forceinline__ void begin(int r, int after) {
     if (!kWalkLookahead) return;   // Z is then read when the row ends
@@ -399,7 +444,7 @@ __global__ void __launch_bounds__(kWideThreads, kFwdCtas)
                    double* __restrict__ closs,
                    const int32_t* __restrict__ order) {
   const int lane = threadIdx.x & 31;
-  FwdVisit vis{colidx, P, Z, D, WITH_DA ? dA : nullptr, pc, 0, lane, 0.0, zero4(), zero4(), -1};
+  FwdVisit vis{colidx, P, Z, D, WITH_DA ? dA : nullptr, pc, 0, lane, 0.0, zero4(), zero4(), -1, -1};
   const int ngroups = (nchunks + kFwdGrab - 1) / kFwdGrab;
   while (true) {
     const int k = next_group(&hdr->work[0], lane);
@@ -420,13 +465,14 @@ __global__ void __launch_bounds__(kWideThreads, kFwdCtas)
 }
 
 // ---- rows and columns without keys -----------------------------------------
-// Rows: D_r = -Z_r and the loss term |Z_r|^2 / 2; columns: G_c = 0.  A warp
+// Rows: the loss term |Z_r|^2 / 2 (their D_r = -Z_r is not stored: no key
+// gathers it); columns: G_c = 0.  A warp
 // takes 32 consecutive rows (columns), finds the empty ones with one ballot
 // and handles them two at a time (half a warp each, one float4 per lane),
 // eight rows in flight.
 __global__ void __launch_bounds__(kWideThreads)
     gnn_empty_kernel(const int32_t* __restrict__ rowptr, int m, const float* __restrict__ Z,
-                     float* __restrict__ D, const int32_t* __restrict__ colptr, int n,
+                     const int32_t* __restrict__ colptr, int n,
                      float* __restrict__ G, WsHeader* hdr, double* partials, double* loss_out) {
   __shared__ double red[kWideWarps];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -469,8 +515,6 @@ __global__ void __launch_bounds__(kWideThreads)
         for (int u = 0; u < 4; ++u) {
           const int k = rr[2 * u + half];
           if (k < 0) continue;
-          reinterpret_cast<float4*>(D + (size_t)(r0 + k) * 64)[sl] =
-              make_float4(-z[u].x, -z[u].y, -z[u].z, -z[u].w);
           lossf += 0.5f * (z[u].x * z[u].x + z[u].y * z[u].y + z[u].z * z[u].z + z[u].w * z[u].w);
         }
       } else {
@@ -586,6 +630,11 @@ struct ColVisit {
   float4 pnext;      // P row of column pnext_c, loaded one column ahead
   int pnext_c;
   float t[kPairs];   // this lane's parts of the batch's dot products
+  int front;         // columns up to this one are prefetched
+
+  __device__ __forceinline__ void ahead(int lo, int pv, int lane_) {
+    if (SDAD_COL_PREFETCH && perm) prefetch_window(P, lo, pv, lane_, &front);
+  }
 
   __device__ __forceinline__ void begin(int c, int after) {
     if (!perm) return;
@@ -646,6 +695,7 @@ __global__ void __launch_bounds__(kWideThreads, kColCtas)
   vis.pcol = zero4();
   vis.pnext = zero4();
   vis.pnext_c = -1;
+  vis.front = -1;
 #pragma unroll
   for (int u = 0; u < kPairs; ++u) vis.t[u] = 0.f;
   const int ngroups = (nchunks + kColGrab - 1) / kColGrab;
@@ -729,10 +779,10 @@ cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const flo
     const int cg = back ? cgroups : 0;
     // mean segments per group: about (segments + groups) / groups
     const GroupWalk w0{A->rowptr, m, kFwdGrab * kWideChunk, fgroups,
-                       (int)std::min<long long>(INT_MAX, 4 * (((long long)m + fgroups + fgroups - 1) / fgroups)),
+                       (int)std::min<long long>(INT_MAX, kOrderHeavy * (((long long)m + fgroups + fgroups - 1) / fgroups)),
                        L.order};
     const GroupWalk w1{A->colptr, n, kColGrab * kWideChunk, cg,
-                       (int)std::min<long long>(INT_MAX, 4 * (((long long)n + cg + std::max(cg, 1) - 1) / std::max(cg, 1))),
+                       (int)std::min<long long>(INT_MAX, kOrderHeavy * (((long long)n + cg + std::max(cg, 1) - 1) / std::max(cg, 1))),
                        L.order + fgroups};
     const int ctas0 = (fgroups + kOrderThreads - 1) / kOrderThreads;
     const int ctas1 = (cg + kOrderThreads - 1) / kOrderThreads;
@@ -747,7 +797,7 @@ cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const flo
   const int ge = std::max(1, std::min((m + n + 255) / 256, sms * 8));
   {
     KTimer t("gnn_empty", st);
-    gnn_empty_kernel<<<ge, kWideThreads, 0, st>>>(A->rowptr, m, Z, L.D, A->colptr, n,
+    gnn_empty_kernel<<<ge, kWideThreads, 0, st>>>(A->rowptr, m, Z, A->colptr, n,
                                                   back ? L.G : nullptr, L.hdr, L.partials, loss);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
