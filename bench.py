@@ -177,9 +177,18 @@ def kernel_bytes(cfg, p, nnz, tmode_csc, want_extra, ranked=False, blocked=0, sp
         b["batax_gram"] = 16 * nnz + 8 * (n + 1) + 8 * jnnz
     elif cfg == "gnn":
         f_in, f_out = 128, 64
+        # rows and columns that hold keys: only their Z, D, P and G rows are walked
+        mr = int(np.count_nonzero(np.bincount(p.row, minlength=m)))
+        nc = int(np.count_nonzero(np.bincount(p.col, minlength=n)))
+        row = 4 * f_out
         b["proj_fwd"] = 4 * n * f_in + 4 * n * f_out + 4 * f_in * f_out
-        b["gnn_fwd"] = 8 * nnz + 4 * (m + 1) + 4 * n * f_out + 4 * m * f_out * 2 + 4 * nnz
-        b["gnn_col"] = 8 * nnz + 4 * (n + 1) + 4 * m * f_out + 4 * n * f_out
+        # pointers; Z of the rows without keys read, G of the columns without keys zeroed
+        b["gnn_empty"] = 4 * (m + 1) + 4 * (n + 1) + row * (m - mr) + row * (n - nc)
+        # keys (index, value); P of each column with keys once; Z read and D written per row with keys
+        b["gnn_fwd"] = 8 * nnz + 4 * (m + 1) + row * nc + 2 * row * mr
+        # keys (index, value, transpose permutation) and dA; D once per row with keys;
+        # P read and G written once per column with keys
+        b["gnn_col"] = 12 * nnz + 4 * nnz + 4 * (n + 1) + row * mr + 2 * row * nc
         b["proj_bwd"] = 4 * n * f_in * 2 + 4 * n * f_out
     return b
 
@@ -213,13 +222,15 @@ NCU_TRAFFIC = {
         "nnz": 67108864,
         "bytes_per_launch": {
             "gnn_col": ("paper_2303_07030_gb300/csrc/k_gnn.cu",
-                        "65d6d51ceb6385902f74447e916ac131e2f74eec", 7444253440 + 1744101888),
+                        "bf50c9d415f5a59ee0ccc2f7e98a7fc141edc82c", 7532439296 + 1790444800),
             "gnn_fwd": ("paper_2303_07030_gb300/csrc/k_gnn.cu",
-                        "65d6d51ceb6385902f74447e916ac131e2f74eec", 5107680256 + 519769856),
+                        "bf50c9d415f5a59ee0ccc2f7e98a7fc141edc82c", 5920281344 + 525560576),
+            "gnn_empty": ("paper_2303_07030_gb300/csrc/k_gnn.cu",
+                          "bf50c9d415f5a59ee0ccc2f7e98a7fc141edc82c", 602441472 + 491051008),
             "proj_bwd": ("paper_2303_07030_gb300/csrc/k_dense.cu",
-                         "7ad6780de9cb33a8892472ffd9057955aca792d8", 3230619392 + 2096632320),
+                         "7ad6780de9cb33a8892472ffd9057955aca792d8", 3228864512 + 2096301824),
             "proj_fwd": ("paper_2303_07030_gb300/csrc/k_dense.cu",
-                         "7ad6780de9cb33a8892472ffd9057955aca792d8", 2150708736 + 1034470144),
+                         "7ad6780de9cb33a8892472ffd9057955aca792d8", 2150849024 + 1033389056),
         },
         "capture": "ncu 1-pass dram bytes of the full workload (one launch per kernel)",
     },

@@ -37,6 +37,18 @@ def test_kernel_bytes_per_config():
     assert bench.step_keys("smmm", q) == q.nnz + q.params["B"][0].size
 
 
+def test_graph_bytes_count_rows_with_keys():
+    # 4 vertices, keys (0,1), (0,2), (2,1): rows 0 and 2 and columns 1 and 2 hold keys
+    row = np.array([0, 0, 2], dtype=np.int32)
+    col = np.array([1, 2, 1], dtype=np.int32)
+    q = W.SparseMatrixProblem("gnn", 4, 4, row, col, np.ones(3, np.float32), {}, {})
+    b = bench.kernel_bytes("gnn", q, 3, True, False)
+    r = 256
+    assert b["gnn_fwd"] == 8 * 3 + 4 * 5 + r * 2 + 2 * r * 2
+    assert b["gnn_col"] == 16 * 3 + 4 * 5 + r * 2 + 2 * r * 2
+    assert b["gnn_empty"] == 4 * 5 * 2 + r * 2 + r * 2
+
+
 def test_names_and_overrides():
     assert bench.transpose_name(0, None) == "CSC"
     assert "2^15" in bench.transpose_name(15, None)
