@@ -222,11 +222,11 @@ NCU_TRAFFIC = {
         "nnz": 67108864,
         "bytes_per_launch": {
             "gnn_col": ("paper_2303_07030_gb300/csrc/k_gnn.cu",
-                        "bf50c9d415f5a59ee0ccc2f7e98a7fc141edc82c", 7532439296 + 1790444800),
+                        "335fd7531fb71576b7e699c4fb0821850d13a572", 7699900672 + 1921329152),
             "gnn_fwd": ("paper_2303_07030_gb300/csrc/k_gnn.cu",
-                        "bf50c9d415f5a59ee0ccc2f7e98a7fc141edc82c", 5920281344 + 525560576),
+                        "335fd7531fb71576b7e699c4fb0821850d13a572", 5918429952 + 525517312),
             "gnn_empty": ("paper_2303_07030_gb300/csrc/k_gnn.cu",
-                          "bf50c9d415f5a59ee0ccc2f7e98a7fc141edc82c", 602441472 + 491051008),
+                          "335fd7531fb71576b7e699c4fb0821850d13a572", 602388992 + 491072000),
             "proj_bwd": ("paper_2303_07030_gb300/csrc/k_dense.cu",
                          "7ad6780de9cb33a8892472ffd9057955aca792d8", 3228864512 + 2096301824),
             "proj_fwd": ("paper_2303_07030_gb300/csrc/k_dense.cu",

@@ -56,6 +56,26 @@ __device__ __forceinline__ float reduce_half8(float (&t)[kPairs], int lane) {
   return x;   // value 4*b3 + 2*b2 + b1 = (sl >> 1) & 7
 }
 
+// The same for four values: returns the half's total of value (sl >> 2) & 3
+// (6 shuffles for the 8 totals of the warp).
+__device__ __forceinline__ float reduce_half4(float (&t)[4], int lane) {
+  const bool b3 = lane & 8, b2 = lane & 4;
+  float u2[2];
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {   // keep values 2*b3 + i, send the other half
+    const float keep = b3 ? t[i + 2] : t[i], send = b3 ? t[i] : t[i + 2];
+    u2[i] = keep + __shfl_xor_sync(FULL_MASK, send, 8);
+  }
+  const float keep = b2 ? u2[1] : u2[0], send = b2 ? u2[0] : u2[1];
+  float x = keep + __shfl_xor_sync(FULL_MASK, send, 4);
+  x += __shfl_xor_sync(FULL_MASK, x, 2);
+  x += __shfl_xor_sync(FULL_MASK, x, 1);
+  return x;   // value 2*b3 + b2 = (sl >> 2) & 3
+}
+
+__device__ __forceinline__ float reduce_half(float (&t)[8], int lane) { return reduce_half8(t, lane); }
+__device__ __forceinline__ float reduce_half(float (&t)[4], int lane) { return reduce_half4(t, lane); }
+
 // The lane holding the total of key offset o (0..15) of a 16-key batch after
 // reduce_half8: key o is pair o / 2 of half o % 2.
 __device__ __forceinline__ int batch_src_lane(int o) { return ((o & 1) << 4) | ((o >> 1) << 1); }

@@ -90,7 +90,7 @@ __device__ __forceinline__ void prefetch_window(const float* X, int lo, int pv, 
 }
 // Resident CTAs per SM the walks are compiled for, and the forward walk's
 // batch: measured fastest with 4 key pairs per batch at 6 CTAs (40
-// registers) for the forward walk, and 8 pairs at 3 CTAs for the column walk
+// registers) for the forward walk, and 4 pairs at 4 CTAs for the column walk
 // (which also holds P_c and the batch's dot products).
 #ifndef SDAD_FWD_CTAS
 #define SDAD_FWD_CTAS 6
@@ -100,12 +100,20 @@ __device__ __forceinline__ void prefetch_window(const float* X, int lo, int pv, 
 #endif
 constexpr int kFwdCtas = SDAD_FWD_CTAS;
 #ifndef SDAD_COL_CTAS
-#define SDAD_COL_CTAS 3
+#define SDAD_COL_CTAS 4
 #endif
 constexpr int kColCtas = SDAD_COL_CTAS;
 // key pairs gathered per batch by the forward walk (the column walk reduces
-// its dot products in batches of kPairs)
+// its dot products in batches of kColPairs)
 constexpr int kFwdPairs = SDAD_FWD_PAIRS;
+// key pairs gathered per batch by the column walk (4 or 8).  Measured on the
+// 2^22-vertex R-MAT graph: 8 pairs at 3 CTAs per SM (76 registers) 2.81 ms,
+// 4 pairs at 4 CTAs (60 registers) 2.74 ms, 4 pairs at 5 CTAs (spills) 3.17 ms.
+#ifndef SDAD_COL_PAIRS
+#define SDAD_COL_PAIRS 4
+#endif
+constexpr int kColPairs = SDAD_COL_PAIRS;
+static_assert(kColPairs == 4 || kColPairs == 8, "the dot-product reductions take 4 or 8 pairs");
 
 __device__ __forceinline__ float2 ld2(const float* base, int r, int lane) {
   return __ldg(reinterpret_cast<const float2*>(base + (size_t)r * 64) + lane);
@@ -629,7 +637,7 @@ struct ColVisit {
   float4 pcol;       // P row of the current column (this lane's elements)
   float4 pnext;      // P row of column pnext_c, loaded one column ahead
   int pnext_c;
-  float t[kPairs];   // this lane's parts of the batch's dot products
+  float t[kColPairs];   // this lane's parts of the batch's dot products
   int front;         // columns up to this one are prefetched
 
   __device__ __forceinline__ void ahead(int lo, int pv, int lane_) {
@@ -658,14 +666,16 @@ struct ColVisit {
   }
   __device__ __forceinline__ void batch_done(int k0, int nk, int lane_) {
     if (!perm) return;
-    const float r = reduce_half8(t, lane_);
-    // lane (h, sl) with sl even holds key k0 + 2 ((sl >> 1) & 7) + h
     const int sl = lane_ & 15;
-    const int kk = k0 + 2 * ((sl >> 1) & 7) + (lane_ >> 4);
+    const float r = reduce_half(t, lane_);
+    // 8 pairs: lane (h, sl) with sl even holds key k0 + 2 ((sl >> 1) & 7) + h;
+    // 4 pairs: lane (h, sl) with sl % 4 == 0 holds key k0 + 2 ((sl >> 2) & 3) + h
+    const int kk = k0 + (lane_ >> 4) + (kColPairs == 8 ? 2 * ((sl >> 1) & 7) : 2 * ((sl >> 2) & 3));
+    const bool holder = kColPairs == 8 ? (sl & 1) == 0 : (sl & 3) == 0;
     const int q = __shfl_sync(FULL_MASK, ql, kk & 31);
-    if ((sl & 1) == 0 && kk < nk) st_stream(dA + q, r);
+    if (holder && kk < nk) st_stream(dA + q, r);
 #pragma unroll
-    for (int u = 0; u < kPairs; ++u) t[u] = 0.f;
+    for (int u = 0; u < kColPairs; ++u) t[u] = 0.f;
   }
   __device__ __forceinline__ void segment(int c, int s0, int s1, float4 tot, int cs, int ce) {
     if (pc.cut(ch, c, s0, s1, cs, ce, tot, lane)) return;
@@ -697,7 +707,7 @@ __global__ void __launch_bounds__(kWideThreads, kColCtas)
   vis.pnext_c = -1;
   vis.front = -1;
 #pragma unroll
-  for (int u = 0; u < kPairs; ++u) vis.t[u] = 0.f;
+  for (int u = 0; u < kColPairs; ++u) vis.t[u] = 0.f;
   const int ngroups = (nchunks + kColGrab - 1) / kColGrab;
   while (true) {
     const int k = next_group(&hdr->work[1], lane);
@@ -709,7 +719,7 @@ __global__ void __launch_bounds__(kWideThreads, kColCtas)
       if (lane == 0) pc.lastseg[ch] = -1;
       __syncwarp();
       vis.ch = ch;
-      if (cs < ce) pair_walk<kPairs>(colptr, n, rowidx, val_csc, D, cs, ce, hint, lane, vis, &hint);
+      if (cs < ce) pair_walk<kColPairs>(colptr, n, rowidx, val_csc, D, cs, ce, hint, lane, vis, &hint);
     }
   }
 }
