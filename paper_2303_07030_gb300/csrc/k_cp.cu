@@ -124,8 +124,18 @@ __global__ void __launch_bounds__(kPipeThreads)
 // Entry-order pass scattering all three factor gradients (outputs zeroed).
 // Eight lanes per entry (four floats each), four entries per warp step;
 // kCpAtomicUnroll steps' index and factor loads are issued together.
-constexpr int kCpAtomicUnroll = 2;
-__global__ void __launch_bounds__(256)
+#ifndef SDAD_CPA_UNROLL
+#define SDAD_CPA_UNROLL 2
+#endif
+// resident CTAs per SM the pass is compiled for: 4 (64 registers) measured
+// 0.966 ms on 10^7 entries, against 0.983 ms at 3 (76 registers) and 1.19 ms
+// at 5 (spills); the grid is the resident CTAs (1.06 ms with 8 CTAs per SM
+// requested and three resident, the rest in a second wave)
+#ifndef SDAD_CPA_MINB
+#define SDAD_CPA_MINB 4
+#endif
+constexpr int kCpAtomicUnroll = SDAD_CPA_UNROLL;
+__global__ void __launch_bounds__(256, SDAD_CPA_MINB)
     cp_atomic_kernel(int nnz, const int32_t* __restrict__ I, const int32_t* __restrict__ J,
                      const int32_t* __restrict__ K, const float* __restrict__ T,
                      const float* __restrict__ A, const float* __restrict__ B,
@@ -195,7 +205,13 @@ cudaError_t run_cp3(const sdad_coo3* T, const float* A, const float* B, const fl
   if (tmode == SDAD_T_ATOMIC) {
     for (int m = 0; m < 3; ++m)
       if (dfac[m] && (e = zero_f32(dfac[m], (size_t)T->dims[m] * 32, st)) != cudaSuccess) return e;
-    const int grid = std::max(1, std::min((nnz + 32 * kCpAtomicUnroll - 1) / (32 * kCpAtomicUnroll), sms * 8));
+    // as many CTAs as are resident at once (a grid-stride loop; no second wave)
+    int per_sm = 1;
+    if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, cp_atomic_kernel, 256, 0)) !=
+        cudaSuccess)
+      return e;
+    const int grid = std::max(1, std::min((nnz + 32 * kCpAtomicUnroll - 1) / (32 * kCpAtomicUnroll),
+                                          sms * std::max(per_sm, 1)));
     {
       KTimer t_cp_atomic("cp_atomic", st);
       cp_atomic_kernel<<<grid, 256, 0, st>>>(nnz, T->idx[0], T->idx[1], T->idx[2], T->val, A, B, C,

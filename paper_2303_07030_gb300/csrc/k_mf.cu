@@ -187,7 +187,34 @@ constexpr size_t kMfSmem = pipe_smem_bytes<2, kMfCap, kMfNS>();
 constexpr int kMfaChunk = kMinCap;   // the piece slots are per kMinCap keys
 constexpr int kMfaThreads = 256;
 constexpr int kMfaWarps = kMfaThreads / 32;
-constexpr int kMfHot = 64;
+#ifndef SDAD_MFA_HOT
+#define SDAD_MFA_HOT 64
+#endif
+constexpr int kMfHot = SDAD_MFA_HOT;
+// key pairs per batch (4 or 8) and resident CTAs per SM the sweep is compiled
+// for.  Measured on 5*10^7 keys: 8 pairs at 3 CTAs (79 registers) 2.83 ms;
+// 8 pairs unbounded (122 registers, 2 CTAs) 3.72 ms; 4 pairs at 4 CTAs 2.93 ms,
+// at 3 CTAs 3.38 ms, unbounded 4.53 ms; 128 hot columns instead of 64: 2.92 ms
+#ifndef SDAD_MFA_PAIRS
+#define SDAD_MFA_PAIRS 8
+#endif
+#ifndef SDAD_MFA_MINB
+#define SDAD_MFA_MINB 3
+#endif
+constexpr int kMfaPairs = SDAD_MFA_PAIRS;
+static_assert(kMfaPairs == 4 || kMfaPairs == 8, "the dot-product reductions take 4 or 8 pairs");
+// after reduce_half over kMfaPairs values: the key offset of the batch whose
+// total lane `lane` holds, whether it is the lane that acts on it, and the
+// lane holding the total of key offset o
+__device__ __forceinline__ int mfa_key_of_lane(int lane) {
+  return kMfaPairs == 8 ? batch_key_of_lane(lane) : 2 * (((lane & 15) >> 2) & 3) + (lane >> 4);
+}
+__device__ __forceinline__ bool mfa_holder(int lane) {
+  return kMfaPairs == 8 ? (lane & 1) == 0 : (lane & 3) == 0;
+}
+__device__ __forceinline__ int mfa_src_lane(int o) {
+  return kMfaPairs == 8 ? batch_src_lane(o) : ((o & 1) << 4) | ((o >> 1) << 2);
+}
 
 __global__ void __launch_bounds__(256)
     mfa_init_kernel(const float* __restrict__ U, const float* __restrict__ V, int m, int n,
@@ -219,7 +246,7 @@ struct MfaPieces {
   int* __restrict__ lastseg;
 };
 
-__global__ void __launch_bounds__(kMfaThreads)
+__global__ void __launch_bounds__(kMfaThreads, SDAD_MFA_MINB)
     mfa_kernel(const int32_t* __restrict__ rowptr, const int32_t* __restrict__ colidx,
                const int32_t* __restrict__ rcolidx, const int32_t* __restrict__ rankcol,
                const float* __restrict__ val, int m, int n, int nnz, int nchunks,
@@ -235,7 +262,7 @@ __global__ void __launch_bounds__(kMfaThreads)
     for (int i = threadIdx.x; i < kMfHot * 64; i += blockDim.x) hot[i] = 0.f;
     __syncthreads();
   }
-  const int kl = batch_key_of_lane(lane);   // the key whose dot product this lane ends with
+  const int kl = mfa_key_of_lane(lane);   // the key whose dot product this lane ends with
   double loss = 0.0;
   // chunks are handed out one at a time from a counter in the workspace
   // header (reset by mfa_init_kernel): hub rows make chunks very unequal
@@ -254,31 +281,31 @@ __global__ void __launch_bounds__(kMfaThreads)
       const int ps = max(s0, cs), pe = min(s1, ce);
       const float4 uv = ld4(U, r, sl);
       float4 acc = zero4();
-      for (int pb = ps; pb < pe; pb += 2 * kPairs) {
-        const int nk = min(2 * kPairs, pe - pb);
+      for (int pb = ps; pb < pe; pb += 2 * kMfaPairs) {
+        const int nk = min(2 * kMfaPairs, pe - pb);
         const bool mine = lane < nk;
         const int jl = mine ? __ldg(colidx + pb + lane) : 0;
         const float al = mine ? __ldg(val + pb + lane) : 0.f;
         const int rk = (ranked && mine) ? __ldg(rcolidx + pb + lane) : INT_MAX;
-        float4 x[kPairs];
-        float t[kPairs];
+        float4 x[kMfaPairs];
+        float t[kMfaPairs];
 #pragma unroll
-        for (int u = 0; u < kPairs; ++u) {
+        for (int u = 0; u < kMfaPairs; ++u) {
           const int kk = 2 * u + h;
           const int j = __shfl_sync(FULL_MASK, jl, kk);
           x[u] = kk < nk ? ld4(V, j, sl) : zero4();
           t[u] = dot4(x[u], uv);
         }
-        const float d = reduce_half8(t, lane);
-        const float e = __shfl_sync(FULL_MASK, al, kl) - d;   // valid where sl is even and kl < nk
-        if ((sl & 1) == 0 && kl < nk) {
+        const float d = reduce_half(t, lane);
+        const float e = __shfl_sync(FULL_MASK, al, kl) - d;   // valid in the holder lanes, kl < nk
+        if (mfa_holder(lane) && kl < nk) {
           loss += (double)e * (double)e;
           if (dR) dR[pb + kl] = 2.f * e;
         }
 #pragma unroll
-        for (int u = 0; u < kPairs; ++u) {
+        for (int u = 0; u < kMfaPairs; ++u) {
           const int kk = 2 * u + h;
-          const float eu = __shfl_sync(FULL_MASK, e, batch_src_lane(kk));
+          const float eu = __shfl_sync(FULL_MASK, e, mfa_src_lane(kk));
           const int j = __shfl_sync(FULL_MASK, jl, kk);
           const int rank = __shfl_sync(FULL_MASK, rk, kk);
           if (kk < nk) {
