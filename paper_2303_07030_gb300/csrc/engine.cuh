@@ -38,6 +38,17 @@ namespace sdad {
 
 constexpr int kConsumerWarps = 8;
 constexpr int kPipeThreads = 32 * (kConsumerWarps + 1);
+// resident CTAs per SM the engine kernels are compiled for (0: no bound; they
+// then take 96 registers, 2 CTAs per SM).  3 CTAs (72 registers, spills)
+// measured slower: MF two passes 4.27 -> 4.74 ms, CP mode pass 0.47 -> 0.51 ms.
+#ifndef SDAD_PIPE_MINB
+#define SDAD_PIPE_MINB 0
+#endif
+#if SDAD_PIPE_MINB > 0
+#define SDAD_PIPE_BOUNDS __launch_bounds__(kPipeThreads, SDAD_PIPE_MINB)
+#else
+#define SDAD_PIPE_BOUNDS __launch_bounds__(kPipeThreads)
+#endif
 
 constexpr int kMaxLong = 32;   // capacity of the per-chunk list of long parts
 constexpr int kSegStage = 128; // segments whose pointers (and side values) are staged

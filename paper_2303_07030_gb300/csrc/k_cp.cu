@@ -109,7 +109,7 @@ struct CpModeBody {
   }
 };
 
-__global__ void __launch_bounds__(kPipeThreads)
+__global__ void SDAD_PIPE_BOUNDS
     cp_mode_kernel(StreamSrc<3> src, CpModeBody body, WsHeader* hdr, double* partials,
                    int first_slot, int finalize, double* loss_out) {
   extern __shared__ __align__(1024) unsigned char smraw[];

@@ -139,7 +139,7 @@ struct MfBody {
   }
 };
 
-__global__ void __launch_bounds__(kPipeThreads)
+__global__ void SDAD_PIPE_BOUNDS
     mf_kernel(StreamSrc<2> src, MfBody body, WsHeader* hdr, double* partials, int first_slot,
               int finalize, double* loss_out) {
   extern __shared__ __align__(1024) unsigned char smraw[];
