@@ -235,12 +235,16 @@ NCU_TRAFFIC = {
         "capture": "ncu 1-pass dram bytes of the full workload (one launch per kernel)",
     },
     "logreg": {
-        # 400,000-row instance, 20,000,407 keys; ranked columns, 2^15-row blocked twin
-        "source": "paper_2303_07030_gb300/csrc/k_scalar.cu",
-        "sha1": "0dbc677f8113ea28c84b7c761a8184b5ebfb8195",
+        # the full workload (49,997,656 keys); ranked columns, 2^15-row blocked twin
         "layout": {"ranked": True, "blocked": 15, "split": False},
-        "bytes_per_key": {"logreg_row": 8.5676, "scalar_bcol": 8.4912},
-        "capture": "ncu capture of the 400k-row instance, scaled by keys",
+        "nnz": 49997656,
+        "bytes_per_launch": {
+            "logreg_row": ("paper_2303_07030_gb300/csrc/k_scalar.cu",
+                           "32e14217d98b55bfc40bba12227a160805b8edbf", 416628992 + 8155392),
+            "scalar_bcol": ("paper_2303_07030_gb300/csrc/k_scalar.cu",
+                            "32e14217d98b55bfc40bba12227a160805b8edbf", 416738560 + 9703680),
+        },
+        "capture": "ncu 1-pass dram bytes of the full workload (one launch per kernel)",
     },
 }
 
@@ -255,23 +259,16 @@ def _sha1(rel):
 
 
 def measured_traffic(cfg, kernel, nnz, layout=None):
-    import hashlib
+    """DRAM bytes per launch of `kernel` from an ncu capture of this very workload
+    (same key count and layout), or (None, None) when none was taken or the
+    kernel's source has changed since (SHA-1 of the file)."""
     ent = NCU_TRAFFIC.get(cfg)
     if ent is None or (ent.get("layout") is not None and layout != ent["layout"]):
         return None, None
-    if "bytes_per_launch" in ent:   # captured on the full workload itself, per kernel
-        got = ent["bytes_per_launch"].get(kernel)
-        if ent.get("nnz") != nnz or got is None or _sha1(got[0]) != got[1]:
-            return None, None
-        return int(got[2]), ent["capture"]
-    try:
-        with open(os.path.join(ROOT, ent["source"]), "rb") as f:
-            if hashlib.sha1(f.read()).hexdigest() != ent["sha1"]:
-                return None, None
-    except OSError:
+    got = ent["bytes_per_launch"].get(kernel)
+    if ent.get("nnz") != nnz or got is None or _sha1(got[0]) != got[1]:
         return None, None
-    b = ent["bytes_per_key"].get(kernel)
-    return (None, None) if b is None else (int(round(b * nnz)), ent["capture"])
+    return int(got[2]), ent["capture"]
 
 
 # ----------------------------------------------------------------------------

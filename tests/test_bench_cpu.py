@@ -87,12 +87,19 @@ def test_flops_and_traffic_tables():
     c = W.make("cp3", "small")
     assert bench.kernel_flops("cp3", c, c.nnz)["cp_atomic"] == 384 * c.nnz
     # a figure is given only for the layout it was captured on
-    lay = dict(bench.NCU_TRAFFIC["logreg"]["layout"])
-    t, src = bench.measured_traffic("logreg", "logreg_row", 1000, lay)
+    ent = bench.NCU_TRAFFIC["logreg"]
+    lay = dict(ent["layout"])
+    t, src = bench.measured_traffic("logreg", "logreg_row", ent["nnz"], lay)
     assert (t is None) == (src is None)
-    lay["blocked"] = 0
+    if t is not None:   # the source file is the one captured
+        assert t == ent["bytes_per_launch"]["logreg_row"][2]
+    # only for the workload it was captured on
     assert bench.measured_traffic("logreg", "logreg_row", 1000, lay) == (None, None)
+    lay["blocked"] = 0
+    assert bench.measured_traffic("logreg", "logreg_row", ent["nnz"], lay) == (None, None)
     assert bench.measured_traffic("lsq", "lsq_row", 1000, None) == (None, None)
+    g = bench.NCU_TRAFFIC["gnn"]
+    assert bench.measured_traffic("gnn", "gnn_col", g["nnz"] + 1, None) == (None, None)
 
 
 def test_default_headline_is_the_largest_workload():
