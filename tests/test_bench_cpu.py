@@ -78,6 +78,13 @@ def test_reference_arm_prints_one_json_line():
     assert d["impl"] == "reference" and d["metric"] == bench.METRIC and d["value"] > 0
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["cpu_baseline"]["kind"] == "oracle"
     assert d["steps"] == 2 and d["warmup"] == 1
+    assert d["cpu_baseline"]["cores"] >= 1.0
+
+
+def test_busy_cores_is_cpu_time_over_wall_time():
+    assert bench.busy_cores(10.0, 10.0) == 1.0
+    assert bench.busy_cores(35.0, 10.0) == 3.5
+    assert bench.busy_cores(0.2, 10.0) == 1.0   # a mostly idle single thread still counts as one
 
 
 def test_flops_and_traffic_tables():
