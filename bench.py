@@ -615,17 +615,27 @@ def measure(cfg, args, ov, dist, world, local, headline, fma):
         kernels[k] = e
 
     # ---------------- end to end: host buffers, copies inside the timing ----
+    # Every step copies its inputs in from pinned host memory, runs, and copies
+    # its loss and gradients back.  Two buffer sets and three streams: while
+    # step s computes, step s + 1's inputs copy in and step s - 1's outputs copy
+    # out (the host link carries both directions at once).  The serial figure
+    # (one stream: in, step, out) is reported beside it.
     e2e = None
     if headline and not args.no_e2e:
         ins = host_inputs(run, cfg)
-        outs = host_outputs(run, cfg)
-        h2d = sum(h.numel() * h.element_size() for _, h in ins)
-        d2h = sum(h.numel() * h.element_size() for _, h in outs)
+        host_in = [h for _, h in ins]
+        run2 = make_run(cfg, p, tmode, ranked, blocked, block_cols)
+        runs = [run, run2]
+        dev_in = [[d for d, _ in ins], list(run2.step_inputs())]
+        outs = [host_outputs(r, cfg) for r in runs]
+        h2d = sum(h.numel() * h.element_size() for h in host_in)
+        d2h = sum(h.numel() * h.element_size() for _, h in outs[0])
+        # serial: one stream
         for _ in range(2):
             for d, h in ins:
                 d.copy_(h, non_blocking=True)
             run.step()
-            for d, h in outs:
+            for d, h in outs[0]:
                 h.copy_(d, non_blocking=True)
         torch.cuda.synchronize()
         barrier()
@@ -636,19 +646,57 @@ def measure(cfg, args, ov, dist, world, local, headline, fma):
             for d, h in ins:
                 d.copy_(h, non_blocking=True)
             run.step()
-            for d, h in outs:
+            for d, h in outs[0]:
                 h.copy_(d, non_blocking=True)
         e1.record(stream)
         torch.cuda.synchronize()
-        run.check()
+        serial_ms = e0.elapsed_time(e1) / args.steps
+        # double-buffered
+        s_in, s_cmp, s_out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+        ev_in = [torch.cuda.Event() for _ in runs]
+        ev_cmp = [torch.cuda.Event() for _ in runs]
+        ev_out = [torch.cuda.Event() for _ in runs]
+
+        def pipelined(first, count):
+            for st in range(first, first + count):
+                b = st % 2
+                if st >= 2:   # step st - 2 has read this set's inputs
+                    s_in.wait_event(ev_cmp[b])
+                with torch.cuda.stream(s_in):
+                    for d, h in zip(dev_in[b], host_in):
+                        d.copy_(h, non_blocking=True)
+                ev_in[b].record(s_in)
+                s_cmp.wait_event(ev_in[b])
+                if st >= 2:   # ... and its outputs are copied out
+                    s_cmp.wait_event(ev_out[b])
+                runs[b].step(s_cmp)
+                ev_cmp[b].record(s_cmp)
+                s_out.wait_event(ev_cmp[b])
+                with torch.cuda.stream(s_out):
+                    for d, h in outs[b]:
+                        h.copy_(d, non_blocking=True)
+                ev_out[b].record(s_out)
+
+        pipelined(0, 2)
+        torch.cuda.synchronize()
+        barrier()
+        e0.record(s_in)
+        pipelined(2, args.steps)
+        e1.record(s_out)   # after the last copy out, which waits for everything before it
+        torch.cuda.synchronize()
+        for r in runs:
+            r.check()
         ems = e0.elapsed_time(e1) / args.steps
         if dist is not None:
-            t = torch.tensor([ems], device="cuda", dtype=torch.float64)
+            t = torch.tensor([ems, serial_ms], device="cuda", dtype=torch.float64)
             dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ems = float(t.item())
+            ems, serial_ms = float(t[0].item()), float(t[1].item())
         e2e = {"value": world * nnz / (ems * 1e-3), "unit": UNIT, "ms_per_step": round(ems, 4),
-               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
-        del ins, outs
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+               "mode": "double-buffered: inputs of step s+1 copy in and outputs of step s-1 copy out "
+                       "while step s runs",
+               "serial_ms_per_step": round(serial_ms, 4)}
+        del ins, outs, run2, runs, dev_in, host_in
     tot = sum(kb.get(k, 0) * v[0] for k, v in per.items()) / max(args.steps, 1)
     res = {
         "value": value, "ms_per_step": round(ms, 5),
