@@ -92,6 +92,7 @@ def parse():
                          "scale); one JSON line with a point per instance")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-jvp", action="store_true", help="skip the forward-mode timing")
     ap.add_argument("--override", action="append", default=[], metavar="KEY=VALUE",
                     help="change a generator parameter of the headline workload (profiling of "
                          "a smaller instance, e.g. m=400000); the line then says so")
@@ -506,6 +507,72 @@ def layout_for(cfg, p, args, S):
     return ranked, blocked, block_cols, split, transpose
 
 
+def jvp_closure(cfg, run, torch):
+    """One forward-mode call of the workload's loss along a seeded tangent of every
+    dense operand and of the sparse values (None for the paper's matrix kernels)."""
+    from paper_2303_07030_gb300 import sdad as S
+    g = torch.Generator(device="cuda")
+    g.manual_seed(20230313)
+
+    def like(t):
+        return torch.randn(t.shape, generator=g, device=t.device, dtype=t.dtype)
+
+    def vals(n):
+        return torch.randn(int(n), generator=g, device="cuda", dtype=torch.float32)
+
+    lt = torch.zeros(1, dtype=torch.float64, device="cuda")
+    if cfg == "lsq":
+        xt, at = like(run.x), vals(run.A.nnz)
+        return lambda: S.sdad_lsq_jvp(run.desc, run.x, run.y, run.loss, lt, xt, at, run.ws)
+    if cfg == "logreg":
+        wt, at = like(run.w), vals(run.X.nnz)
+        return lambda: S.sdad_logreg_jvp(run.desc, run.w, run.y, run.loss, lt, wt, at, run.ws)
+    if cfg == "mf":
+        ut, vt, rt = like(run.U), like(run.V), vals(run.R.nnz)
+        return lambda: S.sdad_mf_jvp(run.desc, run.U, run.V, run.k, run.lam, run.loss, lt, rt,
+                                     ut, vt, run.ws)
+    if cfg == "cp3":
+        at, bt, ct, tt = like(run.A), like(run.B), like(run.C), vals(run.p.nnz)
+        return lambda: S.sdad_cp3_jvp(run.desc, run.A, run.B, run.C, run.R, run.loss, lt, tt,
+                                      at, bt, ct, run.ws)
+    if cfg == "gnn":
+        ht, wt, at = like(run.H), like(run.W), vals(run.A.nnz)
+        return lambda: S.sdad_gnn_jvp(run.desc, run.H, run.W, run.Z, run.f_in, run.f_out,
+                                      run.loss, lt, at, ht, wt, run.ws)
+    return None
+
+
+def time_jvp(cfg, run, nnz, steps, torch, S):
+    """Forward mode (Sec. 4.2): ms per call and keys per second over `steps` calls
+    after three warm-up calls, with the per-kernel times of a bracketed pass."""
+    fn = jvp_closure(cfg, run, torch)
+    if fn is None:
+        return None
+    for _ in range(3):
+        fn()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(steps):
+        fn()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    S.sdad_timing_reset()
+    S.sdad_timing_enable(True)
+    for _ in range(steps):
+        fn()
+    torch.cuda.synchronize()
+    S.sdad_timing_enable(False)
+    per = {}
+    for k, t in S.sdad_timing_records():
+        per.setdefault(k, []).append(t)
+    run.check()
+    return {"ms_per_call": round(ms, 5), "value": nnz / (ms * 1e-3), "unit": UNIT,
+            "tangent": "every dense operand and the sparse values",
+            "kernels": {k: round(sum(v) / len(v), 5) for k, v in per.items()}}
+
+
 def measure(cfg, args, ov, dist, world, local, headline, fma):
     """One workload: timed steps, per-kernel times, rooflines; e2e for the headline."""
     import torch
@@ -697,6 +764,7 @@ def measure(cfg, args, ov, dist, world, local, headline, fma):
                        "while step s runs",
                "serial_ms_per_step": round(serial_ms, 4)}
         del ins, outs, run2, runs, dev_in, host_in
+    jvp = None if args.no_jvp else time_jvp(cfg, run, nnz, min(args.steps, 10), torch, S)
     tot = sum(kb.get(k, 0) * v[0] for k, v in per.items()) / max(args.steps, 1)
     res = {
         "value": value, "ms_per_step": round(ms, 5),
@@ -713,6 +781,7 @@ def measure(cfg, args, ov, dist, world, local, headline, fma):
         "ms_per_step_kernels_bracketed": round(bracketed_ms, 5),
         "gpu_launches": int(len(recs)), "launches_per_step": len(recs) / max(args.steps, 1),
         "hbm_gbs_step": round(tot / (ms * 1e-3) / 1e9, 1), "clocks": clocks, "e2e": e2e,
+        "jvp": jvp,
     }
     del run, flush
     torch.cuda.synchronize()
@@ -835,7 +904,7 @@ def main():
             q, r = measure(c, args, {}, dist, world, local, False, fma)
             del q
             others[c] = {k: r[k] for k in ("value", "ms_per_step", "roofline", "kernels",
-                                           "gpu_launches", "hbm_gbs_step", "clocks")}
+                                           "gpu_launches", "hbm_gbs_step", "clocks", "jvp")}
             others[c]["workload"] = r["config"]["workload"]
             others[c]["nnz"] = r["config"]["nnz"]
             if r["config"]["transpose"]:
@@ -855,7 +924,7 @@ def main():
                 o["gpu_launches"] for o in others.values()),
             "launches_per_step": head["launches_per_step"],
             "hbm_gbs_step": head["hbm_gbs_step"], "clocks": head["clocks"], "e2e": head["e2e"],
-            "cpu_baseline": cpu, "fp32_fma_peak": fma, "configs": others,
+            "cpu_baseline": cpu, "fp32_fma_peak": fma, "jvp": head["jvp"], "configs": others,
         }
         print(json.dumps(line), flush=True)
     if dist is not None:

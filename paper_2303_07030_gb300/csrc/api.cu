@@ -161,6 +161,7 @@ WsLayout ws_layout(int expr, int32_t rows, int32_t cols, int64_t nnz, int32_t wi
     const size_t nch = (size_t)(std::max<int64_t>(nnz, 0) / kMinCap + 2);
     L.closs = reinterpret_cast<double*>(take(sizeof(double) * nch));
     L.order = reinterpret_cast<int32_t*>(take(sizeof(int32_t) * 4 * nch));
+    L.cltan = reinterpret_cast<double*>(take(sizeof(double) * nch));
     L.tfirst = reinterpret_cast<float*>(take(sizeof(float) * nch * f));
     L.tlast = reinterpret_cast<float*>(take(sizeof(float) * nch * f));
   }

@@ -39,6 +39,7 @@ struct WsLayout {
   float* dWpart;      // graph: per-CTA partial H^T G              [kDwParts x f_in x f_out]
   double* closs;      // graph: loss terms of the rows finished inside each chunk [chunks]
   int32_t* order;     // graph: the walks' chunk-group order, then its scratch    [4 x chunks]
+  double* cltan;      // graph, forward mode: the L' terms of the rows finished inside each chunk
   float* tfirst;      // graph, forward mode: pieces of Y' (as pfirst / plast below)
   float* tlast;
   // pieces of segments cut by chunk boundaries (deterministic combination):
@@ -124,6 +125,12 @@ cudaError_t run_gnn_jvp(const sdad_csr* A, const float* H, const float* W, const
 cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const float* Z,
                     double* loss, float* dA, float* dH, float* dW, bool atomic,
                     const WsLayout& L, cudaStream_t st);
+
+// The forward-mode walk over the CSR (graph loss): per chunk, the L and L'
+// terms of its finished rows (L.closs, L.cltan) and the pieces of Y and Y' of
+// its cut rows; hdr->work[0] must be zero on entry.
+cudaError_t run_gnn_jvp_walk(const sdad_csr* A, const float* valt, const float* P,
+                             const float* Pt, const float* Z, const WsLayout& L, cudaStream_t st);
 
 // Dense projection kernels (graph loss): P = H W;  dH = G W^T and per-CTA
 // partials of H^T G;  dW = sum of the partials.

@@ -299,13 +299,18 @@ struct ChunkPieces {
 // 64-wide, float4 per lane, both halves holding the whole row), and
 // vis.key(h, x, q) for every key q (x = the gathered row, held by half h) at
 // the moment the walk is in q's segment.  Segments without keys are skipped
-// (gnn_empty_kernel handles them).
-template <int NP, class Vis>
+// (gnn_empty_kernel handles them).  TAN (forward mode): each key also
+// gathers Xt[idx] (Xt may be NULL: zero) and the segment's tangent
+// ttot = sum of valt * X[idx] + val * Xt[idx] (valt may be NULL: zero) goes
+// to vis.segment2(s, s0, s1, tot, ttot, cs, ce) instead.
+template <int NP, class Vis, bool TAN = false>
 __device__ __forceinline__ void pair_walk(const int32_t* __restrict__ ptr, int nseg,
                                           const int32_t* __restrict__ idx,
                                           const float* __restrict__ val,
                                           const float* __restrict__ X, int cs, int ce, int hint,
-                                          int lane, Vis& vis, int* seg_out) {
+                                          int lane, Vis& vis, int* seg_out,
+                                          const float* __restrict__ valt = nullptr,
+                                          const float* __restrict__ Xt = nullptr) {
   const int h = lane >> 4, sl = lane & 15;
   // the segment holding key cs: the last s with ptr[s] <= cs
   int s = warp_gallop_lower_bound(ptr, hint, nseg + 1, cs + 1) - 1;
@@ -313,57 +318,74 @@ __device__ __forceinline__ void pair_walk(const int32_t* __restrict__ ptr, int n
   vis.front = s;
   vis.begin(s, -1);
   float4 acc = zero4();
+  float4 tacc = zero4();   // TAN only
+  auto close = [&]() {
+    if constexpr (TAN) vis.segment2(s, s0, s1, join_halves(acc), join_halves(tacc), cs, ce);
+    else vis.segment(s, s0, s1, join_halves(acc), cs, ce);
+  };
   for (int base = cs; base < ce; base += 32) {
     const int nk = min(32, ce - base);
     const int jl = lane < nk ? ld_stream(idx + base + lane) : 0;
     const float al = lane < nk ? ld_stream(val + base + lane) : 0.f;
+    float atl = 0.f;
+    if constexpr (TAN) atl = (valt && lane < nk) ? ld_stream(valt + base + lane) : 0.f;
     vis.window(base, nk, lane);
     for (int k0 = 0; k0 < nk; k0 += 2 * NP) {
       float4 x[NP];
+      float4 xt[TAN ? NP : 1];
 #pragma unroll
       for (int u = 0; u < NP; ++u) {
         const int kk = k0 + 2 * u + h;
         const int j = __shfl_sync(FULL_MASK, jl, kk & 31);
         x[u] = kk < nk ? ld4(X, j, sl) : zero4();
+        if constexpr (TAN) xt[u] = (kk < nk && Xt) ? ld4(Xt, j, sl) : zero4();
       }
 #pragma unroll
       for (int u = 0; u < NP; ++u) {
         const int kk = k0 + 2 * u;   // this pair: keys kk (half 0) and kk + 1 (half 1)
         const float a = __shfl_sync(FULL_MASK, al, (kk + h) & 31);
+        float at = 0.f;
+        if constexpr (TAN) at = __shfl_sync(FULL_MASK, atl, (kk + h) & 31);
         if (kk >= nk) break;   // warp-uniform
+        auto add = [&]() {
+          acc = fma4(a, x[u], acc);
+          if constexpr (TAN) tacc = fma4(at, x[u], fma4(a, xt[u], tacc));
+        };
         const int p0 = base + kk;
         const bool two = kk + 1 < nk;
         if ((two ? p0 + 1 : p0) < s1) {   // both keys in segment s (the usual case)
-          acc = fma4(a, x[u], acc);        // an absent second key adds a zero row
+          add();                           // an absent second key adds a zero row
           vis.key(h, x[u], kk + h, u);
           continue;
         }
         // a segment ends inside the pair
         if (p0 >= s1) {
-          vis.segment(s, s0, s1, join_halves(acc), cs, ce);
+          close();
           const Seg g = next_segment(ptr, nseg, s, p0, lane, vis);
           s = g.s; s0 = g.s0; s1 = g.s1;
           vis.begin(s, g.after);
           acc = zero4();
+          tacc = zero4();
         }
-        if (h == 0) acc = fma4(a, x[u], acc);
+        if (h == 0) add();
         vis.key_if(h == 0, x[u], kk, u);
         if (two) {
           if (p0 + 1 >= s1) {
-            vis.segment(s, s0, s1, join_halves(acc), cs, ce);
+            close();
             const Seg g = next_segment(ptr, nseg, s, p0 + 1, lane, vis);
             s = g.s; s0 = g.s0; s1 = g.s1;
             vis.begin(s, g.after);
             acc = zero4();
+            tacc = zero4();
           }
-          if (h == 1) acc = fma4(a, x[u], acc);
+          if (h == 1) add();
           vis.key_if(h == 1, x[u], kk + 1, u);
         }
       }
       vis.batch_done(k0, nk, lane);
     }
   }
-  vis.segment(s, s0, s1, join_halves(acc), cs, ce);
+  close();
   *seg_out = s;
 }
 
@@ -760,6 +782,126 @@ __global__ void __launch_bounds__(kWideThreads)
   }
 }
 
+// Orders the forward walk's fgroups groups of kFwdGrab chunks (the CSR) and,
+// with cgroups > 0, the column walk's (the CSC twin), into L.order.
+static cudaError_t group_order(const sdad_csr* A, int fgroups, int cgroups, const WsLayout& L,
+                               cudaStream_t st) {
+  const int m = A->m, n = A->n, nnz = (int)A->nnz;
+  KTimer t("gnn_order", st);
+  // mean segments per group: about (segments + groups) / groups
+  const GroupWalk w0{A->rowptr, m, kFwdGrab * kWideChunk, fgroups,
+                     (int)std::min<long long>(INT_MAX, kOrderHeavy * (((long long)m + fgroups + fgroups - 1) / fgroups)),
+                     L.order};
+  const GroupWalk w1{A->colptr, n, kColGrab * kWideChunk, cgroups,
+                     (int)std::min<long long>(INT_MAX, kOrderHeavy * (((long long)n + cgroups + std::max(cgroups, 1) - 1) / std::max(cgroups, 1))),
+                     L.order + fgroups};
+  const int ctas0 = (fgroups + kOrderThreads - 1) / kOrderThreads;
+  const int ctas1 = (cgroups + kOrderThreads - 1) / kOrderThreads;
+  int8_t* flag = reinterpret_cast<int8_t*>(L.order + fgroups + cgroups);
+  int32_t* count = L.order + fgroups + cgroups + (fgroups + cgroups + 3) / 4;
+  group_flag_kernel<<<ctas0 + ctas1, kOrderThreads, 0, st>>>(w0, w1, ctas0, nnz, flag, count);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  group_place_kernel<<<ctas0 + ctas1, kOrderThreads, 0, st>>>(w0, w1, ctas0, ctas1, flag, count);
+  return cudaGetLastError();
+}
+
+// ---- forward mode: the walk carrying (Y, Y') --------------------------------
+// Y_r = sum_p val[p] P_j and Y'_r = sum_p (valt[p] P_j + val[p] P'_j); a row
+// finished inside its chunk adds 1/2 |Y_r - Z_r|^2 to L and (Y_r - Z_r) . Y'_r
+// to L' (this chunk's slots); a row cut by chunk boundaries leaves pieces of
+// Y (pfirst / plast) and of Y' (tfirst / tlast).  Same walk, group order and
+// Z prefetch as the reverse-mode forward walk.
+struct JvpVisit {
+  const float* __restrict__ Z;
+  ChunkPieces pc;
+  float* __restrict__ tfirst;
+  float* __restrict__ tlast;
+  int ch, lane;
+  double L, Lt;   // this lane's parts
+  int front;
+
+  __device__ __forceinline__ void ahead(int lo, int pv, int lane_) {
+    if (SDAD_FWD_PREFETCH) prefetch_window(Z, lo, pv, lane_, &front);
+  }
+  __device__ __forceinline__ void begin(int, int) {}
+  __device__ __forceinline__ void window(int, int, int) {}
+  __device__ __forceinline__ void key(int, float4, int, int) {}
+  __device__ __forceinline__ void key_if(bool, float4, int, int) {}
+  __device__ __forceinline__ void batch_done(int, int, int) {}
+  __device__ __forceinline__ void segment2(int r, int s0, int s1, float4 tot, float4 ttot, int cs,
+                                           int ce) {
+    if (pc.cut(ch, r, s0, s1, cs, ce, tot, lane)) {
+      if (lane < 16) st4(s0 < cs ? tfirst : tlast, ch, lane, ttot);
+      return;
+    }
+    const int sl = lane & 15;
+    const float4 z = ld_stream(reinterpret_cast<const float4*>(Z + (size_t)r * 64) + sl);
+    const float4 d = make_float4(tot.x - z.x, tot.y - z.y, tot.z - z.z, tot.w - z.w);
+    if (lane < 16) {
+      L += 0.5 * (double)dot4(d, d);
+      Lt += (double)dot4(d, ttot);
+    }
+  }
+};
+
+#ifndef SDAD_JVP_CTAS
+#define SDAD_JVP_CTAS 4
+#endif
+constexpr int kJvpCtas = SDAD_JVP_CTAS;
+constexpr int kJvpPairs = 4;
+
+__global__ void __launch_bounds__(kWideThreads, kJvpCtas)
+    gnn_jvp_fwd_kernel(const int32_t* __restrict__ rowptr, const int32_t* __restrict__ colidx,
+                       const float* __restrict__ val, const float* __restrict__ valt, int m,
+                       int nnz, int nchunks, const float* __restrict__ P,
+                       const float* __restrict__ Pt, const float* __restrict__ Z, ChunkPieces pc,
+                       float* __restrict__ tfirst, float* __restrict__ tlast, WsHeader* hdr,
+                       double* __restrict__ closs, double* __restrict__ cltan,
+                       const int32_t* __restrict__ order) {
+  const int lane = threadIdx.x & 31;
+  JvpVisit vis{Z, pc, tfirst, tlast, 0, lane, 0.0, 0.0, -1};
+  const int ngroups = (nchunks + kFwdGrab - 1) / kFwdGrab;
+  while (true) {
+    const int k = next_group(&hdr->work[0], lane);
+    if (k >= ngroups) break;   // warp-uniform
+    const int g = __ldg(order + k);
+    int hint = 0;
+    for (int ch = g * kFwdGrab; ch < min((g + 1) * kFwdGrab, nchunks); ++ch) {
+      const int cs = ch * kWideChunk, ce = min(cs + kWideChunk, nnz);
+      if (lane == 0) pc.lastseg[ch] = -1;
+      __syncwarp();
+      vis.ch = ch;
+      vis.L = vis.Lt = 0.0;
+      if (cs < ce)
+        pair_walk<kJvpPairs, JvpVisit, true>(rowptr, m, colidx, val, P, cs, ce, hint, lane, vis,
+                                             &hint, valt, Pt);
+      const double cl = warp_sum_d(vis.L), ct = warp_sum_d(vis.Lt);   // in lane order
+      if (lane == 0) {
+        closs[ch] = cl;
+        cltan[ch] = ct;
+      }
+    }
+  }
+}
+
+cudaError_t run_gnn_jvp_walk(const sdad_csr* A, const float* valt, const float* P,
+                             const float* Pt, const float* Z, const WsLayout& L, cudaStream_t st) {
+  const int nnz = (int)A->nnz;
+  const int nchunks = nnz <= 0 ? 1 : (nnz + kWideChunk - 1) / kWideChunk;
+  const int fgroups = (nchunks + kFwdGrab - 1) / kFwdGrab;
+  cudaError_t e = group_order(A, fgroups, 0, L, st);
+  if (e != cudaSuccess) return e;
+  const int grid = std::max(1, std::min((fgroups + kWideWarps - 1) / kWideWarps,
+                                        device_sm_count() * kJvpCtas));
+  const ChunkPieces pc{L.pfirst, L.plast, L.lastseg};
+  KTimer t("gnn_jvp_walk", st);
+  gnn_jvp_fwd_kernel<<<grid, kWideThreads, 0, st>>>(A->rowptr, A->colidx, A->val, valt, A->m, nnz,
+                                                    nchunks, P, Pt, Z, pc, L.tfirst, L.tlast,
+                                                    L.hdr, L.closs, L.cltan, L.order);
+  return cudaGetLastError();
+}
+
 cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const float* Z,
                     double* loss, float* dA, float* dH, float* dW, bool atomic,
                     const WsLayout& L, cudaStream_t st) {
@@ -784,25 +926,7 @@ cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const flo
   // 1. P = H W
   if ((e = dense_proj_fwd(H, W, L.P, n, L.hdr, st)) != cudaSuccess) return e;
   // the walks' group order
-  {
-    KTimer t("gnn_order", st);
-    const int cg = back ? cgroups : 0;
-    // mean segments per group: about (segments + groups) / groups
-    const GroupWalk w0{A->rowptr, m, kFwdGrab * kWideChunk, fgroups,
-                       (int)std::min<long long>(INT_MAX, kOrderHeavy * (((long long)m + fgroups + fgroups - 1) / fgroups)),
-                       L.order};
-    const GroupWalk w1{A->colptr, n, kColGrab * kWideChunk, cg,
-                       (int)std::min<long long>(INT_MAX, kOrderHeavy * (((long long)n + cg + std::max(cg, 1) - 1) / std::max(cg, 1))),
-                       L.order + fgroups};
-    const int ctas0 = (fgroups + kOrderThreads - 1) / kOrderThreads;
-    const int ctas1 = (cg + kOrderThreads - 1) / kOrderThreads;
-    int8_t* flag = reinterpret_cast<int8_t*>(L.order + fgroups + cg);
-    int32_t* count = L.order + fgroups + cg + (fgroups + cg + 3) / 4;
-    group_flag_kernel<<<ctas0 + ctas1, kOrderThreads, 0, st>>>(w0, w1, ctas0, nnz, flag, count);
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    group_place_kernel<<<ctas0 + ctas1, kOrderThreads, 0, st>>>(w0, w1, ctas0, ctas1, flag, count);
-  }
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if ((e = group_order(A, fgroups, back ? cgroups : 0, L, st)) != cudaSuccess) return e;
   // 2a. rows (and columns) without keys
   const int ge = std::max(1, std::min((m + n + 255) / 256, sms * 8));
   {

@@ -7,12 +7,12 @@
 //   Y_i  = sum_p A_ip P_j,   Y'_i = sum_p (A'_ip P_j + A_ip P'_j)
 //   D_i  = Y_i - Z_i,        L = 1/2 sum_i |D_i|^2,   L' = sum_i D_i . Y'_i
 // Rows without keys add 1/2 |Z_i|^2 to L and nothing to L'.
-// Kernel sequence: P (and P') on the tensor cores; a walk over the CSR (one
-// warp per 1024-key chunk, one key per step, lane l holding elements 2l,
-// 2l+1 of the rows; P_j and P'_j gathered) whose rows finished inside a
-// chunk add their terms and whose rows cut by chunk boundaries leave pieces
-// of Y and Y'; the rows without keys; a fix kernel that completes the cut
-// rows and adds every CTA's sums in a fixed order.  Reproducible bit for bit.
+// Kernel sequence: P (and P') on the tensor cores; the rows without keys; the
+// reverse-mode forward walk's machinery carrying a tangent (run_gnn_jvp_walk
+// in k_gnn.cu: half a warp per key, P_j and P'_j gathered, chunk groups from
+// a work counter in the longest-first order, per-chunk sums of L and L'); a
+// fix kernel that completes the rows cut by chunk boundaries and adds the
+// per-chunk and per-CTA sums in a fixed order.  Reproducible bit for bit.
 #include <algorithm>
 
 #include "common.cuh"
@@ -23,7 +23,6 @@ namespace sdad {
 constexpr int kGjChunk = kMinCap;
 constexpr int kGjThreads = 256;
 constexpr int kGjWarps = kGjThreads / 32;
-constexpr int kGjBatch = 8;        // keys whose rows are gathered before use
 constexpr int kTangentSlots = kMaxPartials / 2;   // L' partials follow L's
 
 __device__ __forceinline__ float2 gj_ld2(const float* base, int r, int lane) {
@@ -31,11 +30,6 @@ __device__ __forceinline__ float2 gj_ld2(const float* base, int r, int lane) {
 }
 __device__ __forceinline__ void gj_st2(float* base, int r, int lane, float2 v) {
   reinterpret_cast<float2*>(base + (size_t)r * 64)[lane] = v;
-}
-__device__ __forceinline__ float gj_wsum(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(FULL_MASK, v, o);
-  return v;
 }
 
 struct GjPieces {
@@ -57,101 +51,35 @@ __device__ __forceinline__ void gj_publish(double L, double Lt, double* partials
   }
 }
 
-__global__ void __launch_bounds__(kGjThreads)
-    gnn_jvp_walk_kernel(const int32_t* __restrict__ rowptr, const int32_t* __restrict__ colidx,
-                        const float* __restrict__ val, const float* __restrict__ valt, int m,
-                        int nnz, int nchunks, const float* __restrict__ P,
-                        const float* __restrict__ Pt, const float* __restrict__ Z, GjPieces pc,
-                        double* partials, int first_slot) {
-  __shared__ double red[kGjWarps];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int gw = blockIdx.x * kGjWarps + warp, nw = gridDim.x * kGjWarps;
-  const int c0 = (int)(((long long)nchunks * gw) / nw), c1 = (int)(((long long)nchunks * (gw + 1)) / nw);
-  double L = 0.0, Lt = 0.0;
-  int hint = 0;
-  for (int ch = c0; ch < c1; ++ch) {
-    const int cs = ch * kGjChunk, ce = min(cs + kGjChunk, nnz);
-    if (lane == 0) pc.lastseg[ch] = -1;
-    __syncwarp();
-    if (cs >= ce) continue;
-    int s = warp_gallop_lower_bound(rowptr, hint, m + 1, cs + 1) - 1;
-    int s0 = __ldg(rowptr + s), s1 = __ldg(rowptr + s + 1);
-    float2 y = make_float2(0.f, 0.f), t = y;
-    // the segment s is done: its terms, or its pieces when a chunk boundary cuts it
-    auto close = [&]() {
-      if (s0 >= cs && s1 <= ce) {
-        const float2 z = gj_ld2(Z, s, lane);
-        const float2 d = make_float2(y.x - z.x, y.y - z.y);
-        L += 0.5 * (double)fmaf(d.x, d.x, d.y * d.y);
-        Lt += (double)fmaf(d.x, t.x, d.y * t.y);
-      } else if (s0 < cs) {
-        gj_st2(pc.yfirst, ch, lane, y);
-        gj_st2(pc.tfirst, ch, lane, t);
-      } else {
-        gj_st2(pc.ylast, ch, lane, y);
-        gj_st2(pc.tlast, ch, lane, t);
-        if (lane == 0) pc.lastseg[ch] = s;
-      }
-    };
-    for (int base = cs; base < ce; base += 32) {
-      const int nk = min(32, ce - base);
-      const int jl = lane < nk ? __ldg(colidx + base + lane) : 0;
-      const float al = lane < nk ? __ldg(val + base + lane) : 0.f;
-      const float atl = (valt && lane < nk) ? __ldg(valt + base + lane) : 0.f;
-      for (int k0 = 0; k0 < nk; k0 += kGjBatch) {
-        float2 x[kGjBatch], xt[kGjBatch];
-#pragma unroll
-        for (int u = 0; u < kGjBatch; ++u) {
-          const int j = __shfl_sync(FULL_MASK, jl, (k0 + u) & 31);
-          const bool ok = k0 + u < nk;
-          x[u] = ok ? gj_ld2(P, j, lane) : make_float2(0.f, 0.f);
-          xt[u] = (ok && Pt) ? gj_ld2(Pt, j, lane) : make_float2(0.f, 0.f);
-        }
-#pragma unroll
-        for (int u = 0; u < kGjBatch; ++u) {
-          const float a = __shfl_sync(FULL_MASK, al, (k0 + u) & 31);
-          const float at = __shfl_sync(FULL_MASK, atl, (k0 + u) & 31);
-          if (k0 + u >= nk) break;   // warp-uniform
-          const int p = base + k0 + u;
-          if (p >= s1) {   // row s is done: move to the row of key p
-            close();
-            s = warp_gallop_lower_bound(rowptr, s + 1, m + 1, p + 1) - 1;
-            s0 = __ldg(rowptr + s);
-            s1 = __ldg(rowptr + s + 1);
-            y = make_float2(0.f, 0.f);
-            t = y;
-          }
-          y.x = fmaf(a, x[u].x, y.x);
-          y.y = fmaf(a, x[u].y, y.y);
-          t.x = fmaf(at, x[u].x, fmaf(a, xt[u].x, t.x));
-          t.y = fmaf(at, x[u].y, fmaf(a, xt[u].y, t.y));
-        }
-      }
-    }
-    close();
-    hint = s;
-  }
-  gj_publish(L, Lt, partials, first_slot + blockIdx.x, red);
-}
-
 // rows without keys: L += 1/2 |Z_r|^2 (one warp per 32 rows)
 __global__ void __launch_bounds__(kGjThreads)
     gnn_jvp_empty_kernel(const int32_t* __restrict__ rowptr, int m, const float* __restrict__ Z,
-                         double* partials) {
+                         WsHeader* hdr, double* partials) {
   __shared__ double red[kGjWarps];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (blockIdx.x == 0 && threadIdx.x == 0) hdr->work[0] = 0;   // the walk's group counter
   const int gw = blockIdx.x * kGjWarps + warp, nw = gridDim.x * kGjWarps;
   double L = 0.0;
   for (int blk = gw; blk < (m + 31) / 32; blk += nw) {
     const int r = blk * 32 + lane;
     const bool e = r < m && __ldg(rowptr + r) == __ldg(rowptr + r + 1);
     unsigned todo = __ballot_sync(FULL_MASK, e);
-    while (todo) {
-      const int k = __ffs(todo) - 1;
-      todo &= todo - 1;
-      const float2 z = gj_ld2(Z, blk * 32 + k, lane);
-      L += 0.5 * (double)gj_wsum(fmaf(z.x, z.x, z.y * z.y)) * (lane == 0 ? 1.0 : 0.0);
+    float lf = 0.f;   // this lane's part (elements 2 lane, 2 lane + 1 of each row), in row order
+    while (todo) {    // warp-uniform: eight rows' loads in flight at a time
+      int rr[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        rr[u] = todo ? __ffs(todo) - 1 : -1;
+        if (todo) todo &= todo - 1;
+      }
+      float2 z[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        z[u] = rr[u] >= 0 ? gj_ld2(Z, blk * 32 + rr[u], lane) : make_float2(0.f, 0.f);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) lf = fmaf(z[u].x, z[u].x, fmaf(z[u].y, z[u].y, lf));
     }
+    L += 0.5 * (double)lf;
   }
   gj_publish(L, 0.0, partials, blockIdx.x, red);
 }
@@ -160,13 +88,19 @@ __global__ void __launch_bounds__(kGjThreads)
 // CTA's sums (slots [0, nslots) of L and of L') in slot order
 __global__ void __launch_bounds__(kGjThreads)
     gnn_jvp_fix_kernel(const int32_t* __restrict__ rowptr, int nchunks, GjPieces pc,
-                       const float* __restrict__ Z, WsHeader* hdr, double* partials,
+                       const float* __restrict__ Z, const double* __restrict__ closs,
+                       const double* __restrict__ cltan, WsHeader* hdr, double* partials,
                        int first_slot, double* loss, double* loss_t) {
   __shared__ double red[kGjWarps];
   __shared__ bool s_last;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int gw = blockIdx.x * kGjWarps + warp, nw = gridDim.x * kGjWarps;
   double L = 0.0, Lt = 0.0;
+  // the walk's per-chunk sums: this CTA adds its own slice, in order
+  for (int ch = blockIdx.x * blockDim.x + threadIdx.x; ch < nchunks; ch += gridDim.x * blockDim.x) {
+    L += closs[ch];
+    Lt += cltan[ch];
+  }
   for (int ch = gw; ch < nchunks; ch += nw) {
     const int s = __ldg(pc.lastseg + ch);
     if (s < 0) continue;   // warp-uniform
@@ -243,22 +177,16 @@ cudaError_t run_gnn_jvp(const sdad_csr* A, const float* H, const float* W, const
   const int ge = std::max(1, std::min((m + 255) / 256, sms * 4));
   {
     KTimer t("gnn_jvp_empty", st);
-    gnn_jvp_empty_kernel<<<ge, kGjThreads, 0, st>>>(A->rowptr, m, Z, L.partials);
+    gnn_jvp_empty_kernel<<<ge, kGjThreads, 0, st>>>(A->rowptr, m, Z, L.hdr, L.partials);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
-  const int gw = std::max(1, std::min((nchunks + kGjWarps - 1) / kGjWarps, sms * 8));
-  {
-    KTimer t("gnn_jvp_walk", st);
-    gnn_jvp_walk_kernel<<<gw, kGjThreads, 0, st>>>(A->rowptr, A->colidx, A->val, valt, m, nnz,
-                                                    nchunks, L.P, Pt, Z, pc, L.partials, ge);
-  }
-  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if ((e = run_gnn_jvp_walk(A, valt, L.P, Pt, Z, L, st)) != cudaSuccess) return e;
   const int gf = std::max(1, std::min((nchunks + kGjWarps - 1) / kGjWarps, sms * 4));
-  static_assert(kTangentSlots >= 152 * 16, "partial slots of the three kernels");
+  static_assert(kTangentSlots >= 152 * 8, "partial slots of the empty and fix kernels");
   {
     KTimer t("gnn_jvp_fix", st);
-    gnn_jvp_fix_kernel<<<gf, kGjThreads, 0, st>>>(A->rowptr, nchunks, pc, Z, L.hdr, L.partials,
-                                                   ge + gw, loss, loss_t);
+    gnn_jvp_fix_kernel<<<gf, kGjThreads, 0, st>>>(A->rowptr, nchunks, pc, Z, L.closs, L.cltan,
+                                                   L.hdr, L.partials, ge, loss, loss_t);
   }
   return cudaGetLastError();
 }
