@@ -136,6 +136,9 @@ cudaError_t run_gnn_jvp_walk(const sdad_csr* A, const float* valt, const float* 
 // partials of H^T G;  dW = sum of the partials.
 cudaError_t dense_proj_fwd(const float* H, const float* W, float* P, int n, WsHeader* hdr,
                            cudaStream_t st);
+// P = H W + H2 W2 in one sweep (the forward mode's P' = H' W + H W')
+cudaError_t dense_proj_fwd2(const float* H, const float* W, const float* H2, const float* W2,
+                            float* P, int n, WsHeader* hdr, cudaStream_t st);
 cudaError_t dense_proj_bwd(const float* H, const float* W, const float* G, float* dH,
                            float* dWpart, float* dW, int n, WsHeader* hdr, cudaStream_t st);
 

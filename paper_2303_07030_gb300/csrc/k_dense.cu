@@ -59,9 +59,12 @@ constexpr uint32_t kGRow = kFout * 4;   // ... of G
 constexpr uint32_t kFwdRaw = 0;                         // 2 stages x 64 rows of H (fp32)
 constexpr uint32_t kFwdRawStage = kHalfM * kHRow;       // 32 KB
 constexpr uint32_t kFwdA = kFwdRaw + 2 * kFwdRawStage;  // [hi|lo][kb] x kBlk
-constexpr uint32_t kFwdW = kFwdA + 4 * kBlk;            // W^T: [hi|lo][kb] x 64 rows x 128 B
-constexpr uint32_t kFwdBar = kFwdW + 4 * 64 * 128;
-constexpr uint32_t kFwdSmem = kFwdBar + 64 + 1024;      // barriers, the TMEM slot, alignment
+constexpr uint32_t kFwdW = kFwdA + 4 * kBlk;            // W^T: [hi|lo][kb] x 64 rows x 128 B, per source
+constexpr uint32_t kFwdWBytes = 4 * 64 * 128;
+// NSRC sources (P = H W, or P = H W + H2 W2): barriers after the NSRC W^T
+constexpr uint32_t fwd_bar(int nsrc) { return kFwdW + (uint32_t)nsrc * kFwdWBytes; }
+constexpr uint32_t fwd_smem(int nsrc) { return fwd_bar(nsrc) + 64 + 1024; }   // + barriers, TMEM slot, alignment
+constexpr uint32_t kFwdSmem = fwd_smem(1);
 // shared-memory map of proj_bwd_kernel
 constexpr uint32_t kBwdRawStage = kHalfM * (kHRow + kGRow);   // 48 KB: 64 rows of H, then of G
 constexpr uint32_t kBwdRaw = 0;
@@ -70,7 +73,7 @@ constexpr uint32_t kBwdH = kBwdG + 2 * kBlk;            // [hi|lo][block] x kBlk
 constexpr uint32_t kBwdW = kBwdH + 4 * kBlk;            // W: [hi|lo] x kBlk
 constexpr uint32_t kBwdBar = kBwdW + 2 * kBlk;
 constexpr uint32_t kBwdSmem = kBwdBar + 64 + 1024;
-static_assert(kFwdSmem <= 227 * 1024 && kBwdSmem <= 227 * 1024, "shared memory of one CTA");
+static_assert(fwd_smem(2) <= 227 * 1024 && kBwdSmem <= 227 * 1024, "shared memory of one CTA");
 
 __device__ __forceinline__ uint32_t bf2_bits(__nv_bfloat162 v) {
   return *reinterpret_cast<const uint32_t*>(&v);
@@ -190,45 +193,58 @@ struct RawRing {
 };
 
 // ---------------------------------------------------------------------------
-// P = H W
+// P = H W  (NSRC = 1), or P = H W + H2 W2  (NSRC = 2: the forward mode's
+// P' = H' W + H W' as one product; both sources' rows of a tile go through the
+// same raw stages and split buffers, one after the other, and their MMAs add
+// into the tile's accumulator)
 // ---------------------------------------------------------------------------
+template <int NSRC>
 __global__ void __launch_bounds__(kDenseThreads, 1)
     proj_fwd_kernel(const float* __restrict__ H, const float* __restrict__ W,
+                    const float* __restrict__ H2, const float* __restrict__ W2,
                     float* __restrict__ P, int n, WsHeader* hdr) {
   extern __shared__ unsigned char dense_smem[];
   const uint32_t base = align1024(smem_u32(dense_smem));
   unsigned char* gbase = dense_smem + (base - smem_u32(dense_smem));
-  uint64_t* full = reinterpret_cast<uint64_t*>(gbase + kFwdBar);
+  uint64_t* full = reinterpret_cast<uint64_t*>(gbase + fwd_bar(NSRC));
   uint64_t* mma = full + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + kFwdBar + 24);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(gbase + fwd_bar(NSRC) + 24);
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   constexpr uint32_t idesc = tc::idesc_bf16(kTileM, kFout, false, false);
   auto A = [&](int part, int kb) { return base + kFwdA + (uint32_t)(part * 2 + kb) * kBlk; };
-  auto Wt = [&](int part, int kb) { return base + kFwdW + (uint32_t)(part * 2 + kb) * (64 * 128); };
+  auto Wt = [&](int src, int part, int kb) {
+    return base + kFwdW + (uint32_t)src * kFwdWBytes + (uint32_t)(part * 2 + kb) * (64 * 128);
+  };
   auto raw = [&](int h) { return base + kFwdRaw + (uint32_t)h * kFwdRawStage; };
 
   const int ntiles = (n + kTileM - 1) / kTileM;
   const int grid = gridDim.x;
   const int nloc = (ntiles - (int)blockIdx.x + grid - 1) / grid;   // >= 1: grid <= tiles
+  // half h of source q of local tile i into raw stage h
+  auto issue = [&](int i, int q, int h) {
+    const int r0 = ((int)blockIdx.x + i * grid) * kTileM + h * kHalfM;
+    const uint32_t bytes = (uint32_t)half_rows(r0, n) * kHRow;
+    mbar_arrive_expect_tx(&full[h], bytes);
+    if (bytes) bulk_load(raw(h), (q == 0 ? H : H2) + (size_t)r0 * kFin, bytes, smem_u32(&full[h]));
+  };
   RawRing ring{full, {0, 0}, {0, 0}};
   if (tid == 0) {
     mbar_init(&full[0], 1);
     mbar_init(&full[1], 1);
     mbar_init(mma, 1);
     fence_mbar_init();
-    for (int h = 0; h < 2; ++h) {   // tile 0's halves
-      const int r0 = (int)blockIdx.x * kTileM + h * kHalfM;
-      const uint32_t bytes = (uint32_t)half_rows(r0, n) * kHRow;
-      mbar_arrive_expect_tx(&full[h], bytes);
-      if (bytes) bulk_load(raw(h), H + (size_t)r0 * kFin, bytes, smem_u32(&full[h]));
-    }
+    for (int h = 0; h < 2; ++h) issue(0, 0, h);   // tile 0's halves of the first source
   }
   ring.n_issued[0] = ring.n_issued[1] = 1;
   if (warp == 0) tc::tmem_alloc(tmem_slot, 2 * kFout);   // two accumulators of 64 columns
-  // operand B = W^T (row n' = column n' of W), once per CTA
-  for (int idx = tid; idx < kFin * kFout; idx += kDenseThreads) {
-    const int k = idx / kFout, nn = idx % kFout;
-    put1(Wt(0, k >> 6), Wt(1, k >> 6), tc::sw128_offset_b16(nn, k & 63), __ldg(W + idx));
+  // operand B = W^T (row n' = column n' of W) of each source, once per CTA
+#pragma unroll
+  for (int q = 0; q < NSRC; ++q) {
+    const float* Wq = q == 0 ? W : W2;
+    for (int idx = tid; idx < kFin * kFout; idx += kDenseThreads) {
+      const int k = idx / kFout, nn = idx % kFout;
+      put1(Wt(q, 0, k >> 6), Wt(q, 1, k >> 6), tc::sw128_offset_b16(nn, k & 63), __ldg(Wq + idx));
+    }
   }
   tc::fence_proxy_async_smem();
   tc::fence_before_sync();
@@ -238,49 +254,54 @@ __global__ void __launch_bounds__(kDenseThreads, 1)
 
   const int q4 = warp & 3, cg = warp >> 2;   // epilogue: TMEM lanes 32 q4.., columns 16 cg..
   bool ok = true;
-  int last = -1;   // local index of the last tile whose MMAs were issued
-  for (int i = 0; i < nloc; ++i) {
+  int last = -1;      // local index of the last tile whose MMAs were issued
+  int ncommit = 0;    // MMA groups committed so far (one per tile and source)
+  for (int i = 0; i < nloc && ok; ++i) {
     const int t = (int)blockIdx.x + i * grid, row0 = t * kTileM;
-    if (i >= 1) {   // the split parts are free once tile i-1's MMAs are done
-      ok = __syncthreads_and(mbar_wait(mma, (uint32_t)((i - 1) & 1), hdr));
-      if (!ok) break;
-      tc::fence_after_sync();
-    }
-    for (int h = 0; h < 2; ++h) {
-      ok = __syncthreads_and(mbar_wait(&full[h], ring.parity(h), hdr));
-      if (!ok) break;
-      ++ring.n_waited[h];
-      split_half<32>(raw(h), A(0, 0), A(1, 0), h * kHalfM, half_rows(row0 + h * kHalfM, n));
-      __syncthreads();   // the stage is read: refill it with the next tile's half
-      if (i + 1 < nloc) {
-        if (tid == 0) {
-          const int r0 = row0 + grid * kTileM + h * kHalfM;
-          const uint32_t bytes = (uint32_t)half_rows(r0, n) * kHRow;
-          mbar_arrive_expect_tx(&full[h], bytes);
-          if (bytes) bulk_load(raw(h), H + (size_t)r0 * kFin, bytes, smem_u32(&full[h]));
-        }
-        ++ring.n_issued[h];
+#pragma unroll 1
+    for (int q = 0; q < NSRC; ++q) {
+      if (ncommit > 0) {   // the split parts are free once the last MMA group is done
+        ok = __syncthreads_and(mbar_wait(mma, (uint32_t)((ncommit - 1) & 1), hdr));
+        if (!ok) break;
+        tc::fence_after_sync();
       }
+      for (int h = 0; h < 2; ++h) {
+        ok = __syncthreads_and(mbar_wait(&full[h], ring.parity(h), hdr));
+        if (!ok) break;
+        ++ring.n_waited[h];
+        split_half<32>(raw(h), A(0, 0), A(1, 0), h * kHalfM, half_rows(row0 + h * kHalfM, n));
+        __syncthreads();   // the stage is read: refill it with the next source's half, or the next tile's
+        const bool more = q + 1 < NSRC || i + 1 < nloc;
+        if (more) {
+          if (tid == 0) {
+            if (q + 1 < NSRC) issue(i, q + 1, h);
+            else issue(i + 1, 0, h);
+          }
+          ++ring.n_issued[h];
+        }
+      }
+      if (!ok) break;
+      tc::fence_proxy_async_smem();
+      tc::fence_before_sync();
+      __syncthreads();
+      if (tid == 0) {
+        tc::fence_after_sync();
+        const uint32_t d = tmem + (uint32_t)(kFout * (i & 1));
+#pragma unroll
+        for (int kb = 0; kb < 2; ++kb)
+#pragma unroll
+          for (int s = 0; s < 4; ++s) {
+            const uint64_t ah = kdesc(A(0, kb), s), al = kdesc(A(1, kb), s);
+            const uint64_t bh = kdesc(Wt(q, 0, kb), s), bl = kdesc(Wt(q, 1, kb), s);
+            tc::mma_bf16(d, ah, bh, idesc, q > 0 || (kb | s) != 0);
+            tc::mma_bf16(d, ah, bl, idesc, true);
+            tc::mma_bf16(d, al, bh, idesc, true);
+          }
+        tc::mma_commit(mma);
+      }
+      ++ncommit;
     }
     if (!ok) break;
-    tc::fence_proxy_async_smem();
-    tc::fence_before_sync();
-    __syncthreads();
-    if (tid == 0) {
-      tc::fence_after_sync();
-      const uint32_t d = tmem + (uint32_t)(kFout * (i & 1));
-#pragma unroll
-      for (int kb = 0; kb < 2; ++kb)
-#pragma unroll
-        for (int s = 0; s < 4; ++s) {
-          const uint64_t ah = kdesc(A(0, kb), s), al = kdesc(A(1, kb), s);
-          const uint64_t bh = kdesc(Wt(0, kb), s), bl = kdesc(Wt(1, kb), s);
-          tc::mma_bf16(d, ah, bh, idesc, (kb | s) != 0);
-          tc::mma_bf16(d, ah, bl, idesc, true);
-          tc::mma_bf16(d, al, bh, idesc, true);
-        }
-      tc::mma_commit(mma);
-    }
     last = i;
     if (i >= 1) {   // tile i-1's accumulator to P while the tensor cores work on tile i
       const int row = (t - grid) * kTileM + 32 * q4 + lane;
@@ -289,7 +310,7 @@ __global__ void __launch_bounds__(kDenseThreads, 1)
     }
   }
   if (ok && last >= 0) {
-    ok = __syncthreads_and(mbar_wait(mma, (uint32_t)(last & 1), hdr));
+    ok = __syncthreads_and(mbar_wait(mma, (uint32_t)((ncommit - 1) & 1), hdr));
     if (ok) {
       tc::fence_after_sync();
       const int row = ((int)blockIdx.x + last * grid) * kTileM + 32 * q4 + lane;
@@ -298,7 +319,7 @@ __global__ void __launch_bounds__(kDenseThreads, 1)
     }
   }
   if (!ok) {   // a wait gave up: let the issued copies land and the MMAs end
-    if (last >= 0) mbar_drain(mma, (uint32_t)(last & 1), hdr);
+    if (ncommit > 0) mbar_drain(mma, (uint32_t)((ncommit - 1) & 1), hdr);
     ring.drain(hdr);
   }
   tc::fence_before_sync();
@@ -480,11 +501,24 @@ int dense_grid(int n) {
 
 cudaError_t dense_proj_fwd(const float* H, const float* W, float* P, int n, WsHeader* hdr,
                            cudaStream_t st) {
-  cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void*>(proj_fwd_kernel), (int)kFwdSmem);
+  cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void*>(proj_fwd_kernel<1>), (int)kFwdSmem);
   if (e != cudaSuccess || n <= 0) return e;
   {
     KTimer t("proj_fwd", st);
-    proj_fwd_kernel<<<dense_grid(n), kDenseThreads, kFwdSmem, st>>>(H, W, P, n, hdr);
+    proj_fwd_kernel<1><<<dense_grid(n), kDenseThreads, kFwdSmem, st>>>(H, W, nullptr, nullptr, P,
+                                                                       n, hdr);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t dense_proj_fwd2(const float* H, const float* W, const float* H2, const float* W2,
+                            float* P, int n, WsHeader* hdr, cudaStream_t st) {
+  constexpr uint32_t smem = fwd_smem(2);
+  cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void*>(proj_fwd_kernel<2>), (int)smem);
+  if (e != cudaSuccess || n <= 0) return e;
+  {
+    KTimer t("proj_fwd2", st);
+    proj_fwd_kernel<2><<<dense_grid(n), kDenseThreads, smem, st>>>(H, W, H2, W2, P, n, hdr);
   }
   return cudaGetLastError();
 }

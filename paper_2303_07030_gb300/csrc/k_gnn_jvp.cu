@@ -142,14 +142,6 @@ __global__ void __launch_bounds__(kGjThreads)
   }
 }
 
-__global__ void add_rows_kernel(float4* __restrict__ a, const float4* __restrict__ b, size_t n4) {
-  for (size_t i = blockIdx.x * (size_t)blockDim.x + threadIdx.x; i < n4;
-       i += (size_t)gridDim.x * blockDim.x) {
-    const float4 x = a[i], y = __ldg(b + i);
-    a[i] = make_float4(x.x + y.x, x.y + y.y, x.z + y.z, x.w + y.w);
-  }
-}
-
 cudaError_t run_gnn_jvp(const sdad_csr* A, const float* H, const float* W, const float* Z,
                         const float* valt, const float* Ht, const float* Wt, double* loss,
                         double* loss_t, const WsLayout& L, cudaStream_t st) {
@@ -157,21 +149,13 @@ cudaError_t run_gnn_jvp(const sdad_csr* A, const float* H, const float* W, const
   const int m = A->m, n = A->n, nnz = (int)A->nnz;
   const int nchunks = nnz <= 0 ? 1 : (nnz + kGjChunk - 1) / kGjChunk;
   cudaError_t e;
-  // P = H W; P' = H' W + H W' (in the G buffer; H W' first goes to D)
+  // P = H W; P' = H' W + H W' (in the G buffer), one sweep over H' and H
   if ((e = dense_proj_fwd(H, W, L.P, n, L.hdr, st)) != cudaSuccess) return e;
   const float* Pt = nullptr;
-  if (Ht && (e = dense_proj_fwd(Ht, W, L.G, n, L.hdr, st)) != cudaSuccess) return e;
-  if (Wt) {
-    if ((e = dense_proj_fwd(H, Wt, Ht ? L.D : L.G, n, L.hdr, st)) != cudaSuccess) return e;
-    if (Ht && n > 0) {
-      const size_t n4 = (size_t)n * 16;
-      const int g = (int)std::max<size_t>(1, std::min<size_t>((n4 + 255) / 256, (size_t)sms * 8));
-      KTimer t("gnn_jvp_add", st);
-      add_rows_kernel<<<g, 256, 0, st>>>(reinterpret_cast<float4*>(L.G),
-                                         reinterpret_cast<const float4*>(L.D), n4);
-      if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    }
-  }
+  if (Ht && Wt) e = dense_proj_fwd2(Ht, W, H, Wt, L.G, n, L.hdr, st);
+  else if (Ht) e = dense_proj_fwd(Ht, W, L.G, n, L.hdr, st);
+  else if (Wt) e = dense_proj_fwd(H, Wt, L.G, n, L.hdr, st);
+  if (e != cudaSuccess) return e;
   if (Ht || Wt) Pt = L.G;
   const GjPieces pc{L.pfirst, L.plast, L.tfirst, L.tlast, L.lastseg};
   const int ge = std::max(1, std::min((m + 255) / 256, sms * 4));

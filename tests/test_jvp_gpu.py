@@ -252,7 +252,7 @@ def test_mf_cp3_jvp_full_size():
 
 
 # ----------------------------------------------------------------------------
-# graph propagation: P' = H' W + H W' on the tensor cores, Y' = A' P + A P'
+# graph propagation: P' = H' W + H W' on the tensor cores (one two-source product), Y' = A' P + A P'
 # ----------------------------------------------------------------------------
 
 def _jvp_gnn(run, valt, Ht, Wt):
@@ -320,11 +320,12 @@ def test_gnn_jvp_zero_tangent_and_empty_rows():
 def test_gnn_jvp_full_size():
     p = W.make("gnn", "full")
     rng = np.random.default_rng(17)
-    valt, _, Wt = _gnn_tangents(rng, p)
+    valt, Ht, Wt = _gnn_tangents(rng, p)
     run = R.GnnRun(p)
-    L, Lt = _jvp_gnn(run, valt, None, Wt)
+    # every tangent: P' = H' W + H W' as one two-source product
+    L, Lt = _jvp_gnn(run, valt, Ht, Wt)
     d = p.dense
-    ref = oracle.gnn_jvp(p.m, p.n, p.row, p.col, p.val, d["H"], d["W"], d["Z"], valt, None, Wt)
+    ref = oracle.gnn_jvp(p.m, p.n, p.row, p.col, p.val, d["H"], d["W"], d["Z"], valt, Ht, Wt)
     g = oracle.gnn(p.m, p.n, p.row, p.col, p.val, d["H"], d["W"], d["Z"])
     assert abs(L - ref["loss"]) <= TOL * abs(ref["loss"])
-    assert abs(Lt - ref["loss_t"]) <= TOL * _sbound([(g["dA"], valt), (g["dW"], Wt)])
+    assert abs(Lt - ref["loss_t"]) <= TOL * _sbound([(g["dA"], valt), (g["dH"], Ht), (g["dW"], Wt)])
