@@ -14,6 +14,7 @@
 #include <algorithm>
 
 #include "common.cuh"
+#include "halfwarp.cuh"
 #include "internal.h"
 
 namespace sdad {
@@ -144,15 +145,22 @@ __device__ __forceinline__ float4 mul4f(const float4& a, const float4& b) {
   return make_float4(a.x * b.x, a.y * b.y, a.z * b.z, a.w * b.w);
 }
 
-// Matrix factorisation, k = 64: a warp takes 1024-key chunks of R (CSR),
-// four keys per step, eight lanes per key (eight of the 64 factor entries
-// each); each group follows its key's row through the chunk.  Per key
+// Matrix factorisation, k = 64: a warp takes 1024-key chunks of R (CSR), row
+// by row; U_i and U'_i are loaded once per row (half a warp holds a row, one
+// float4 per lane), and the row's keys go eight at a time, half a warp per
+// key: V_j and V'_j gathered, the eight dot products of each kind reduced
+// together.  Per key
 //   e = R - U_i . V_j,  e' = R' - (U'_i . V_j + U_i . V'_j),  L += e^2, L' += 2 e e'.
 // Then the regulariser over the dense factors: lam (|U|^2 + |V|^2) and its
-// tangent 2 lam (U . U' + V . V').
+// tangent 2 lam (U . U' + V . V').  Per-lane sums in a fixed order:
+// reproducible.
 constexpr int kMfJvpChunk = 1024;
+constexpr int kMfJvpPairs = 4;   // key pairs per batch
+#ifndef SDAD_MFJVP_MINB
+#define SDAD_MFJVP_MINB 3
+#endif
 
-__global__ void __launch_bounds__(kJvpThreads)
+__global__ void __launch_bounds__(kJvpThreads, SDAD_MFJVP_MINB)
     mf_jvp_kernel(const int32_t* __restrict__ rowptr, const int32_t* __restrict__ colidx,
                   const float* __restrict__ val, const float* __restrict__ valt, int m, int n,
                   int nnz, const float* __restrict__ U, const float* __restrict__ V,
@@ -160,45 +168,55 @@ __global__ void __launch_bounds__(kJvpThreads)
                   WsHeader* hdr, double* partials, double* loss, double* loss_t) {
   __shared__ double red[kJvpWarps];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int slot = lane >> 3, sl = lane & 7;
+  const int h = lane >> 4, sl = lane & 15;
   const int gw = blockIdx.x * kJvpWarps + warp, nw = gridDim.x * kJvpWarps;
   const int nchunks = (nnz + kMfJvpChunk - 1) / kMfJvpChunk;
+  // after reduce_half over four values: lane (h, sl) with sl % 4 == 0 holds
+  // the total of key 2 ((sl >> 2) & 3) + h of the batch
+  const int kl = 2 * ((sl >> 2) & 3) + h;
+  const bool holder = (sl & 3) == 0;
   double L = 0.0, Lt = 0.0;
   for (int ch = gw; ch < nchunks; ch += nw) {   // warp-uniform
-    const int ks = ch * kMfJvpChunk, ke = min(ks + kMfJvpChunk, nnz);
-    int rg = warp_lower_bound(rowptr, 0, m + 1, ks + 1) - 1;   // the row of key ks
-    int eg = __ldg(rowptr + rg + 1);
-    for (int base = ks; base < ke; base += 4) {
-      const int p = base + slot;
-      const bool act = p < ke;
-      while (act && p >= eg) {   // this group's key is in a later row
-        ++rg;
-        eg = __ldg(rowptr + rg + 1);
+    const int cs = ch * kMfJvpChunk, ce = min(cs + kMfJvpChunk, nnz);
+    int r = warp_lower_bound(rowptr, 0, m + 1, cs + 1) - 1;   // the row of key cs
+    int s0 = __ldg(rowptr + r), s1 = __ldg(rowptr + r + 1);
+    while (true) {
+      const int ps = max(s0, cs), pe = min(s1, ce);
+      const float4 uv = ld4(U, r, sl);
+      const float4 ut = Ut ? ld4(Ut, r, sl) : zero4();
+      for (int pb = ps; pb < pe; pb += 2 * kMfJvpPairs) {
+        const int nk = min(2 * kMfJvpPairs, pe - pb);
+        const bool mine = lane < nk;
+        const int jl = mine ? __ldg(colidx + pb + lane) : 0;
+        const float al = mine ? __ldg(val + pb + lane) : 0.f;
+        const float atl = (mine && valt) ? __ldg(valt + pb + lane) : 0.f;
+        float4 x[kMfJvpPairs], xt[kMfJvpPairs];
+#pragma unroll
+        for (int u = 0; u < kMfJvpPairs; ++u) {
+          const int kk = 2 * u + h;
+          const int j = __shfl_sync(FULL_MASK, jl, kk);
+          x[u] = kk < nk ? ld4(V, j, sl) : zero4();
+          xt[u] = (kk < nk && Vt) ? ld4(Vt, j, sl) : zero4();
+        }
+        float t[kMfJvpPairs], tt[kMfJvpPairs];
+#pragma unroll
+        for (int u = 0; u < kMfJvpPairs; ++u) {
+          t[u] = dot4(x[u], uv);
+          tt[u] = dot4(x[u], ut) + dot4(xt[u], uv);
+        }
+        const float d = reduce_half(t, lane), dt = reduce_half(tt, lane);
+        const float e = __shfl_sync(FULL_MASK, al, kl) - d;
+        const float et = __shfl_sync(FULL_MASK, atl, kl) - dt;
+        if (holder && kl < nk) {
+          L += (double)e * (double)e;
+          Lt += 2.0 * (double)e * (double)et;
+        }
       }
-      float4 u0 = make_float4(0.f, 0.f, 0.f, 0.f), u1 = u0, v0 = u0, v1 = u0;
-      float4 ut0 = u0, ut1 = u0, vt0 = u0, vt1 = u0;
-      float r = 0.f, rt = 0.f;
-      if (act) {
-        const int j = __ldg(colidx + p);
-        r = __ldg(val + p);
-        rt = valt ? __ldg(valt + p) : 0.f;
-        u0 = ld4(U, rg, 64, 2 * sl);
-        u1 = ld4(U, rg, 64, 2 * sl + 1);
-        v0 = ld4(V, j, 64, 2 * sl);
-        v1 = ld4(V, j, 64, 2 * sl + 1);
-        ut0 = ld4z(Ut, rg, 64, 2 * sl);
-        ut1 = ld4z(Ut, rg, 64, 2 * sl + 1);
-        vt0 = ld4z(Vt, j, 64, 2 * sl);
-        vt1 = ld4z(Vt, j, 64, 2 * sl + 1);
-      }
-      const float d = group_sum<8>(dot4f(u0, v0) + dot4f(u1, v1));
-      const float dt = group_sum<8>(dot4f(ut0, v0) + dot4f(ut1, v1) + dot4f(u0, vt0) +
-                                    dot4f(u1, vt1));
-      if (act && sl == 0) {
-        const float e = r - d, et = rt - dt;
-        L += (double)e * (double)e;
-        Lt += 2.0 * (double)e * (double)et;
-      }
+      if (s1 >= ce) break;
+      // the next row with keys: the one holding key s1
+      r = warp_gallop_lower_bound(rowptr, r + 1, m + 1, s1 + 1) - 1;
+      s0 = __ldg(rowptr + r);
+      s1 = __ldg(rowptr + r + 1);
     }
   }
   // regulariser
@@ -268,9 +286,15 @@ cudaError_t run_mf_jvp(const sdad_csr* R, const float* U, const float* V, float 
                        const float* valt, const float* Ut, const float* Vt, double* loss,
                        double* loss_t, const WsLayout& L, cudaStream_t st) {
   const int nchunks = (int)((R->nnz + kMfJvpChunk - 1) / kMfJvpChunk);
+  // as many CTAs as are resident at once (the chunks are strided over the warps)
+  int per_sm = 1;
+  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, mf_jvp_kernel,
+                                                                kJvpThreads, 0);
+  if (e != cudaSuccess) return e;
   const int grid = std::max(1, std::min(std::max((nchunks + kJvpWarps - 1) / kJvpWarps,
                                                  (R->m + R->n + 255) / 256),
-                                        std::min(device_sm_count() * 8, kMaxPartials / 2)));
+                                        std::min(device_sm_count() * std::max(per_sm, 1),
+                                                 kMaxPartials / 2)));
   {
     KTimer t("mf_jvp", st);
     mf_jvp_kernel<<<grid, kJvpThreads, 0, st>>>(R->rowptr, R->colidx, R->val, valt, R->m, R->n,
