@@ -223,15 +223,15 @@ NCU_TRAFFIC = {
         "nnz": 67108864,
         "bytes_per_launch": {
             "gnn_col": ("paper_2303_07030_gb300/csrc/k_gnn.cu",
-                        "335fd7531fb71576b7e699c4fb0821850d13a572", 7699900672 + 1921329152),
+                        "1df2e0ce72d0e526498cc03569641c1fcdeeb879", 7699332352 + 1920760832),
             "gnn_fwd": ("paper_2303_07030_gb300/csrc/k_gnn.cu",
-                        "335fd7531fb71576b7e699c4fb0821850d13a572", 5918429952 + 525517312),
+                        "1df2e0ce72d0e526498cc03569641c1fcdeeb879", 5918758144 + 525570816),
             "gnn_empty": ("paper_2303_07030_gb300/csrc/k_gnn.cu",
-                          "335fd7531fb71576b7e699c4fb0821850d13a572", 602388992 + 491072000),
+                          "1df2e0ce72d0e526498cc03569641c1fcdeeb879", 602359040 + 491017728),
             "proj_bwd": ("paper_2303_07030_gb300/csrc/k_dense.cu",
-                         "7ad6780de9cb33a8892472ffd9057955aca792d8", 3228864512 + 2096301824),
+                         "b83192d0b63745197114a081c7ba70ebb98cbf5d", 3229664512 + 2096571392),
             "proj_fwd": ("paper_2303_07030_gb300/csrc/k_dense.cu",
-                         "7ad6780de9cb33a8892472ffd9057955aca792d8", 2150849024 + 1033389056),
+                         "b83192d0b63745197114a081c7ba70ebb98cbf5d", 2150552832 + 1033324544),
         },
         "capture": "ncu 1-pass dram bytes of the full workload (one launch per kernel)",
     },
@@ -241,9 +241,9 @@ NCU_TRAFFIC = {
         "nnz": 49997656,
         "bytes_per_launch": {
             "logreg_row": ("paper_2303_07030_gb300/csrc/k_scalar.cu",
-                           "32e14217d98b55bfc40bba12227a160805b8edbf", 416628992 + 8155392),
+                           "27511a24b3fadccf241b92a0236303fc2a5a640e", 416612352 + 8102912),
             "scalar_bcol": ("paper_2303_07030_gb300/csrc/k_scalar.cu",
-                            "32e14217d98b55bfc40bba12227a160805b8edbf", 416738560 + 9703680),
+                            "27511a24b3fadccf241b92a0236303fc2a5a640e", 416723200 + 9714944),
         },
         "capture": "ncu 1-pass dram bytes of the full workload (one launch per kernel)",
     },

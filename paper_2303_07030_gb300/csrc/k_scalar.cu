@@ -754,7 +754,11 @@ cudaError_t launch_rows(const char* name, const Op& op, const sdad_csr* A, const
                         double* loss, double scale, float* dA, float* dxa, float* rvec,
                         const WsLayout& L, cudaStream_t st) {
   const int nblk = (A->m + 31) / 32;
-  int grid = std::max(1, (nblk + kRowWarps * kRowBlocksPerWarp - 1) / (kRowWarps * kRowBlocksPerWarp));
+  // blocks of 32 rows per warp: two on large matrices; one when that leaves
+  // fewer warps than the GPU holds (a small matrix is latency-bound: more
+  // warps, fewer dependent round trips each)
+  const int bpw = nblk >= device_sm_count() * 64 * kRowBlocksPerWarp ? kRowBlocksPerWarp : 1;
+  int grid = std::max(1, (nblk + kRowWarps * bpw - 1) / (kRowWarps * bpw));
   grid = std::min(grid, kMaxPartials);
   {
     KTimer t(name, st);
