@@ -7,7 +7,8 @@
  * Expressions: five losses (least squares, logistic regression, matrix
  * factorisation, CP decomposition, graph propagation), the paper's matrix
  * kernels SMVM, SMMM and BATAX (gradients, and BATAX's Jacobian), and the
- * forward mode of four losses (the directional derivative along a tangent).
+ * forward mode of the five losses (the directional derivative along a
+ * tangent).
  *
  * Semantics follow Shaikhha, Huot, Hashemian, "Differentiable Programming for
  * Sparse Tensors" (arXiv 2303.07030):
@@ -473,7 +474,8 @@ sdad_status sdad_cp3_jvp(const sdad_coo3* T, const float* A, const float* B, con
  *   L = 1/2 |A (H W) - Z|^2 and its directional derivative L' along a tangent
  *   of A's values (A_t_val on keys(A), CSR order), of H (H_t, n x 128) and of
  *   W (W_t, 128 x 64), by the tensorized forward rules of Sec. 4.2 with a
- *   real tangent: P' = H' W + H W' (tensor cores, as P), Y' = A' P + A P',
+ *   real tangent: P' = H' W + H W' (one two-source tensor-core product),
+ *   Y' = A' P + A P',
  *   L' = sum_i (Y_i - Z_i) . Y'_i.  Every tangent is nullable (zero); dense
  *   arrays 16-byte aligned.  One pass over the CSR (no CSC twin needed).
  *   Workspace: as sdad_gnn_grad.  Reproducible bit for bit.
