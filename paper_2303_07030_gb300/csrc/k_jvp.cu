@@ -308,8 +308,15 @@ cudaError_t run_cp3_jvp(const sdad_coo3* T, const float* A, const float* B, cons
                         const float* Tt, const float* At, const float* Bt, const float* Ct,
                         double* loss, double* loss_t, const WsLayout& L, cudaStream_t st) {
   const int nnz = (int)T->nnz;
+  // as many CTAs as are resident at once (a grid-stride loop over uniform
+  // entries: a second wave only lengthens the tail)
+  int per_sm = 1;
+  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, cp3_jvp_kernel,
+                                                                kJvpThreads, 0);
+  if (e != cudaSuccess) return e;
   const int grid = std::max(1, std::min((nnz + 31) / 32,
-                                        std::min(device_sm_count() * 8, kMaxPartials / 2)));
+                                        std::min(device_sm_count() * std::max(per_sm, 1),
+                                                 kMaxPartials / 2)));
   {
     KTimer t("cp3_jvp", st);
     cp3_jvp_kernel<<<grid, kJvpThreads, 0, st>>>(nnz, T->idx[0], T->idx[1], T->idx[2], T->val,
