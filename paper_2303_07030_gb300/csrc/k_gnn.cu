@@ -2,11 +2,13 @@
 //
 // Kernel sequence of one call:
 //   1. P = H W                                           (dense projection)
-//   2. rows without keys: their loss term |Z_r|^2 / 2 (columns without
-//      keys: G_c = 0), then, in the walks' group order, the forward walk over the CSR (one warp per
-//      1024-key chunk): Y_r = sum_p val[p] P[colidx[p]];  rows finished inside
-//      the chunk: D_r = Y_r - Z_r, loss += |D_r|^2 / 2, dA[p] = D_r . P[colidx[p]];
-//      rows cut by chunk boundaries: one 64-wide piece per chunk
+//   2. the walks' chunk-group order (most segments first); rows without
+//      keys: their loss term |Z_r|^2 / 2 (columns without keys: G_c = 0);
+//      then the forward walk over the CSR (a warp per group of two 1024-key
+//      chunks, groups taken from a work counter): Y_r = sum_p val[p]
+//      P[colidx[p]];  rows finished inside the chunk: D_r = Y_r - Z_r,
+//      loss += |D_r|^2 / 2, dA[p] = D_r . P[colidx[p]];  rows cut by chunk
+//      boundaries: one 64-wide piece per chunk
 //   3. fix: D_r of the cut rows from their pieces (chunk order), loss terms
 //   4. dA of the cut rows' keys, chunk by chunk (hub rows are spread over many)
 //   5. G = A^T D: the same walk over the CSC twin, gathering D; cut columns
@@ -20,11 +22,12 @@
 // Lane layout of the walks: a warp takes two keys at a time, one per half
 // warp; lane l of half h = l / 16 holds elements 4(l % 16) .. 4(l % 16) + 3
 // of the 64-wide rows, so one warp instruction gathers two 256-byte rows with
-// 16-byte loads.  Sixteen keys (eight pairs) are gathered before they are
-// used.  Each half keeps its own partial sum of the open segment; a segment
+// 16-byte loads.  A batch of key pairs (four in both walks) is gathered
+// before it is used.  Each half keeps its own partial sum of the open segment; a segment
 // that ends is closed by adding the two halves (one shuffle of a float4), so
 // every sum has a fixed order (chunk structure, lane layout) and the results
-// are reproducible.
+// are reproducible.  The forward mode's walk (gnn_jvp_fwd_kernel, near the
+// end) is the forward walk carrying a tangent.
 #include <algorithm>
 #include <climits>
 
