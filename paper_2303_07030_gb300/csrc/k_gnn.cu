@@ -177,8 +177,9 @@ __device__ __forceinline__ int next_group(uint32_t* ctr, int lane) {
 // without a vertex permutation puts them at the high numbers) the groups
 // handed out last were the slowest, and a few warps ran on long after the
 // others.  So the groups that meet at least four times the mean number of
-// segments are handed out first, the others after them; both keep their
-// matrix order, so the warps in flight still work on neighbouring groups,
+// segments are handed out first (the forward walk's chunk by chunk, so that
+// a group of light rows is walked by two warps), the others after them; both
+// keep their matrix order, so the warps in flight still work on neighbouring groups,
 // which share more of their gathered rows in L2 (sorting all groups by
 // their segment count made the column walk a seventh slower).  The order
 // changes no result: every chunk writes its own slots, which the fix kernels
@@ -193,7 +194,10 @@ struct GroupWalk {   // one walk's groups, for the order kernels
   const int32_t* ptr;   // segment pointers (rowptr or colptr)
   int nseg, keys, ngroups;
   int thr;              // segments that make a group heavy
-  int32_t* order;       // [ngroups]
+  int grab;             // chunks per group
+  bool split;           // hand a heavy group out chunk by chunk
+  int32_t* order;       // [ngroups + heavy groups when split]: items, see group_place_kernel
+  int32_t* nitems;      // the number of items (NULL: ngroups, no split)
 };
 
 // CTA b orders groups [1024 b', 1024 b' + 1024) of walk 0 (b' = b) or of walk
@@ -271,8 +275,16 @@ __global__ void __launch_bounds__(kOrderThreads)
   for (int i = 0; i < warp; ++i) rank += part[i][0];
   if (g < w.ngroups) {
     const int hrank = hbefore + rank;                        // heavy groups before g
-    w.order[heavy ? hrank : hall + (g - hrank)] = g;
+    if (!w.split) {
+      w.order[heavy ? hrank : hall + (g - hrank)] = g;
+    } else if (heavy) {   // one item per chunk: -1 - c for chunk c
+      const int c0 = g * w.grab;
+      for (int u = 0; u < w.grab; ++u) w.order[w.grab * hrank + u] = -1 - (c0 + u);
+    } else {
+      w.order[w.grab * hall + (g - hrank)] = g;
+    }
   }
+  if (w.nitems && b == 0 && t == 0) *w.nitems = w.ngroups + (w.split ? (w.grab - 1) * hall : 0);
 }
 
 struct ChunkPieces {
@@ -475,16 +487,18 @@ __global__ void __launch_bounds__(kWideThreads, kFwdCtas)
                    const float* __restrict__ P, const float* __restrict__ Z, float* __restrict__ D,
                    float* __restrict__ dA, ChunkPieces pc, WsHeader* hdr,
                    double* __restrict__ closs,
-                   const int32_t* __restrict__ order) {
+                   const int32_t* __restrict__ order, const int32_t* __restrict__ order_items) {
   const int lane = threadIdx.x & 31;
   FwdVisit vis{colidx, P, Z, D, WITH_DA ? dA : nullptr, pc, 0, lane, 0.0, zero4(), zero4(), -1, -1};
-  const int ngroups = (nchunks + kFwdGrab - 1) / kFwdGrab;
+  const int nitems = __ldg(order_items);
   while (true) {
     const int k = next_group(&hdr->work[0], lane);
-    if (k >= ngroups) break;   // warp-uniform
-    const int g = __ldg(order + k);
+    if (k >= nitems) break;   // warp-uniform
+    const int e = __ldg(order + k);   // a group, or -1 - c for chunk c alone
+    const int c0 = e >= 0 ? e * kFwdGrab : -1 - e;
+    const int c1 = e >= 0 ? min(c0 + kFwdGrab, nchunks) : c0 + 1;
     int hint = 0;
-    for (int ch = g * kFwdGrab; ch < min((g + 1) * kFwdGrab, nchunks); ++ch) {
+    for (int ch = c0; ch < c1; ++ch) {
       const int cs = ch * kWideChunk, ce = min(cs + kWideChunk, nnz);
       if (lane == 0) pc.lastseg[ch] = -1;
       __syncwarp();
@@ -786,22 +800,33 @@ __global__ void __launch_bounds__(kWideThreads)
 }
 
 // Orders the forward walk's fgroups groups of kFwdGrab chunks (the CSR) and,
-// with cgroups > 0, the column walk's (the CSC twin), into L.order.
+// with cgroups > 0, the column walk's (the CSC twin).  Layout in L.order:
+// the forward walk's items [2 fgroups at most], the column walk's groups
+// [cgroups], the flags, the per-CTA counts, and the forward walk's item count.
+struct WalkOrder {
+  const int32_t* fwd;     // items: a group g >= 0, or -1 - c for chunk c alone
+  const int32_t* nitems;  // ... their number (device)
+  const int32_t* col;     // groups of the column walk
+};
 static cudaError_t group_order(const sdad_csr* A, int fgroups, int cgroups, const WsLayout& L,
-                               cudaStream_t st) {
+                               cudaStream_t st, WalkOrder* out) {
   const int m = A->m, n = A->n, nnz = (int)A->nnz;
   KTimer t("gnn_order", st);
+  const int ctas0 = (fgroups + kOrderThreads - 1) / kOrderThreads;
+  const int ctas1 = (cgroups + kOrderThreads - 1) / kOrderThreads;
+  int32_t* ord0 = L.order;
+  int32_t* ord1 = L.order + 2 * (size_t)fgroups;
+  int8_t* flag = reinterpret_cast<int8_t*>(ord1 + cgroups);
+  int32_t* count = ord1 + cgroups + (fgroups + cgroups + 3) / 4;
+  int32_t* nitems = count + ctas0 + ctas1;
   // mean segments per group: about (segments + groups) / groups
   const GroupWalk w0{A->rowptr, m, kFwdGrab * kWideChunk, fgroups,
                      (int)std::min<long long>(INT_MAX, kOrderHeavy * (((long long)m + fgroups + fgroups - 1) / fgroups)),
-                     L.order};
+                     kFwdGrab, true, ord0, nitems};
   const GroupWalk w1{A->colptr, n, kColGrab * kWideChunk, cgroups,
                      (int)std::min<long long>(INT_MAX, kOrderHeavy * (((long long)n + cgroups + std::max(cgroups, 1) - 1) / std::max(cgroups, 1))),
-                     L.order + fgroups};
-  const int ctas0 = (fgroups + kOrderThreads - 1) / kOrderThreads;
-  const int ctas1 = (cgroups + kOrderThreads - 1) / kOrderThreads;
-  int8_t* flag = reinterpret_cast<int8_t*>(L.order + fgroups + cgroups);
-  int32_t* count = L.order + fgroups + cgroups + (fgroups + cgroups + 3) / 4;
+                     kColGrab, false, ord1, nullptr};
+  *out = WalkOrder{ord0, nitems, ord1};
   group_flag_kernel<<<ctas0 + ctas1, kOrderThreads, 0, st>>>(w0, w1, ctas0, nnz, flag, count);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
@@ -861,16 +886,19 @@ __global__ void __launch_bounds__(kWideThreads, kJvpCtas)
                        const float* __restrict__ Pt, const float* __restrict__ Z, ChunkPieces pc,
                        float* __restrict__ tfirst, float* __restrict__ tlast, WsHeader* hdr,
                        double* __restrict__ closs, double* __restrict__ cltan,
-                       const int32_t* __restrict__ order) {
+                       const int32_t* __restrict__ order,
+                       const int32_t* __restrict__ order_items) {
   const int lane = threadIdx.x & 31;
   JvpVisit vis{Z, pc, tfirst, tlast, 0, lane, 0.0, 0.0, -1};
-  const int ngroups = (nchunks + kFwdGrab - 1) / kFwdGrab;
+  const int nitems = __ldg(order_items);
   while (true) {
     const int k = next_group(&hdr->work[0], lane);
-    if (k >= ngroups) break;   // warp-uniform
-    const int g = __ldg(order + k);
+    if (k >= nitems) break;   // warp-uniform
+    const int e = __ldg(order + k);   // a group, or -1 - c for chunk c alone
+    const int c0 = e >= 0 ? e * kFwdGrab : -1 - e;
+    const int c1 = e >= 0 ? min(c0 + kFwdGrab, nchunks) : c0 + 1;
     int hint = 0;
-    for (int ch = g * kFwdGrab; ch < min((g + 1) * kFwdGrab, nchunks); ++ch) {
+    for (int ch = c0; ch < c1; ++ch) {
       const int cs = ch * kWideChunk, ce = min(cs + kWideChunk, nnz);
       if (lane == 0) pc.lastseg[ch] = -1;
       __syncwarp();
@@ -893,7 +921,8 @@ cudaError_t run_gnn_jvp_walk(const sdad_csr* A, const float* valt, const float* 
   const int nnz = (int)A->nnz;
   const int nchunks = nnz <= 0 ? 1 : (nnz + kWideChunk - 1) / kWideChunk;
   const int fgroups = (nchunks + kFwdGrab - 1) / kFwdGrab;
-  cudaError_t e = group_order(A, fgroups, 0, L, st);
+  WalkOrder wo;
+  cudaError_t e = group_order(A, fgroups, 0, L, st, &wo);
   if (e != cudaSuccess) return e;
   const int grid = std::max(1, std::min((fgroups + kWideWarps - 1) / kWideWarps,
                                         device_sm_count() * kJvpCtas));
@@ -901,7 +930,7 @@ cudaError_t run_gnn_jvp_walk(const sdad_csr* A, const float* valt, const float* 
   KTimer t("gnn_jvp_walk", st);
   gnn_jvp_fwd_kernel<<<grid, kWideThreads, 0, st>>>(A->rowptr, A->colidx, A->val, valt, A->m, nnz,
                                                     nchunks, P, Pt, Z, pc, L.tfirst, L.tlast,
-                                                    L.hdr, L.closs, L.cltan, L.order);
+                                                    L.hdr, L.closs, L.cltan, wo.fwd, wo.nitems);
   return cudaGetLastError();
 }
 
@@ -929,7 +958,8 @@ cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const flo
   // 1. P = H W
   if ((e = dense_proj_fwd(H, W, L.P, n, L.hdr, st)) != cudaSuccess) return e;
   // the walks' group order
-  if ((e = group_order(A, fgroups, back ? cgroups : 0, L, st)) != cudaSuccess) return e;
+  WalkOrder wo;
+  if ((e = group_order(A, fgroups, back ? cgroups : 0, L, st, &wo)) != cudaSuccess) return e;
   // 2a. rows (and columns) without keys
   const int ge = std::max(1, std::min((m + n + 255) / 256, sms * 8));
   {
@@ -943,7 +973,8 @@ cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const flo
     KTimer t("gnn_fwd", st);
     auto fwd = (dA && !dA_in_col) ? gnn_fwd_kernel<true> : gnn_fwd_kernel<false>;
     fwd<<<gf1, kWideThreads, 0, st>>>(A->rowptr, A->colidx, A->val, m, nnz, nchunks, L.P, Z, L.D,
-                                      dA_in_col ? nullptr : dA, pc, L.hdr, L.closs, L.order);
+                                      dA_in_col ? nullptr : dA, pc, L.hdr, L.closs, wo.fwd,
+                                      wo.nitems);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   // 3. cut rows (also finalises the loss over every partial slot)
@@ -979,7 +1010,7 @@ cudaError_t run_gnn(const sdad_csr* A, const float* H, const float* W, const flo
     gnn_col_kernel<<<gc1, kWideThreads, 0, st>>>(A->colptr, A->rowidx, A->val_csc, n, nnz,
                                                   nchunks, L.D, L.G, pc,
                                                   dA_in_col ? A->csc_perm : nullptr, L.P, dA,
-                                                  L.hdr, L.order + fgroups);
+                                                  L.hdr, wo.col);
   }
   if ((e = cudaGetLastError()) != cudaSuccess) return e;
   {
