@@ -223,15 +223,15 @@ NCU_TRAFFIC = {
         "nnz": 67108864,
         "bytes_per_launch": {
             "gnn_col": ("paper_2303_07030_gb300/csrc/k_gnn.cu",
-                        "1df2e0ce72d0e526498cc03569641c1fcdeeb879", 7699332352 + 1920760832),
+                        "dd3221af39633b7b53b0c1a2bd68e53ef5b27e88", 7699289856 + 1921465088),
             "gnn_fwd": ("paper_2303_07030_gb300/csrc/k_gnn.cu",
-                        "1df2e0ce72d0e526498cc03569641c1fcdeeb879", 5918758144 + 525570816),
+                        "dd3221af39633b7b53b0c1a2bd68e53ef5b27e88", 5900874496 + 521272832),
             "gnn_empty": ("paper_2303_07030_gb300/csrc/k_gnn.cu",
-                          "1df2e0ce72d0e526498cc03569641c1fcdeeb879", 602359040 + 491017728),
+                          "dd3221af39633b7b53b0c1a2bd68e53ef5b27e88", 602373888 + 490958592),
             "proj_bwd": ("paper_2303_07030_gb300/csrc/k_dense.cu",
-                         "b83192d0b63745197114a081c7ba70ebb98cbf5d", 3229664512 + 2096571392),
+                         "b83192d0b63745197114a081c7ba70ebb98cbf5d", 3229915904 + 2096727040),
             "proj_fwd": ("paper_2303_07030_gb300/csrc/k_dense.cu",
-                         "b83192d0b63745197114a081c7ba70ebb98cbf5d", 2150552832 + 1033324544),
+                         "b83192d0b63745197114a081c7ba70ebb98cbf5d", 2150839552 + 1033744128),
         },
         "capture": "ncu 1-pass dram bytes of the full workload (one launch per kernel)",
     },
