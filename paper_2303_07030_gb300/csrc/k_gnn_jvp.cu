@@ -28,9 +28,6 @@ constexpr int kTangentSlots = kMaxPartials / 2;   // L' partials follow L's
 __device__ __forceinline__ float2 gj_ld2(const float* base, int r, int lane) {
   return __ldg(reinterpret_cast<const float2*>(base + (size_t)r * 64) + lane);
 }
-__device__ __forceinline__ void gj_st2(float* base, int r, int lane, float2 v) {
-  reinterpret_cast<float2*>(base + (size_t)r * 64)[lane] = v;
-}
 
 struct GjPieces {
   float* __restrict__ yfirst;   // [chunks x 64]: parts of Y of a row begun earlier
